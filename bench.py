@@ -1,0 +1,438 @@
+#!/usr/bin/env python3
+"""Throughput of the GB300 retrieval hot path: queries/s at top-k and the
+fraction of the roofline reached by the dominant kernel.
+
+Default workload (one step = one search call): the paper-shaped dense top-5
+search, 32768 chunks x 768 bf16, a batch of 256 queries (Sec. 5.1 shapes:
+32K chunks, 768-d embeddings).  --config/--batch select the other workloads
+(0 tiny fp32, 2 clustered 4096 queries, 3 hybrid 1024 queries, 4 scale 1M
+chunks with a 4096-row upsert before each 2048-query search).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Timing: W untimed steps, then K steps; before every step a 512 MiB buffer is
+written (L2 flush, outside the timed events); each step is bracketed by CUDA
+events on the launch stream; the library's own events time the search kernel
+itself for the roofline.  Under torchrun every rank runs the same workload on
+its own GPU (replicas), the slowest rank's time counts and `value` adds the
+queries of all ranks.  --impl reference times the CPU oracle on the host cores
+(bounded samples of the same workload).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2608_08340_gb300 import workloads  # noqa: E402
+
+L2_FLUSH_BYTES = 512 << 20
+KERNEL_SOURCES = ["common.cuh", "search_tc.cuh", "search_simt.cuh", "merge.cu", "bm25.cu",
+                  "upsert.cu"]
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--config", type=int, default=1)
+    p.add_argument("--batch", type=int, default=None)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+def default_batch(cfg: int) -> int:
+    return {0: 16, 1: 256, 2: 4096, 3: 1024, 4: 2048}[cfg]
+
+
+def workload_name(cfg: int, w) -> str:
+    base = {0: "tiny dense top-5", 1: "paper-shaped dense top-5", 2: "clustered dense top-10",
+            3: "hybrid dense+BM25 top-5", 4: "scale dense top-100 with 4096-row upserts"}[cfg]
+    return f"{base}: {w.n} x {w.d} {w.dtype}, {w.q} queries/step"
+
+
+def roofline_terms(w, cfg):
+    """Algorithmic bytes and flops of one search-kernel launch."""
+    elem = 4 if w.dtype == "f32" else 2
+    corpus = w.n * w.d * elem
+    queries = w.q * w.d * elem
+    nbytes = corpus + queries
+    if cfg == 3:
+        nbytes += w.q * ((w.n + 3) // 4 * 4) * 4      # fused epilogue reads the BM25 block
+    flops = 2.0 * w.q * w.n * w.d
+    return nbytes, flops
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            m = json.load(f)
+        return float(m["hbm_gbs"]), float(m["bf16_tflops"]), "measured"
+    return 6800.0, 1900.0, "fallback"
+
+
+def source_hash() -> str:
+    h = hashlib.sha256()
+    for name in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, "paper_2608_08340_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def ncu_traffic(workload_key: str):
+    """DRAM bytes per launch of the dominant kernel from the committed ncu
+    summary, if it was taken on the current kernel sources."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        table = json.load(f)
+    ent = table.get(workload_key)
+    if not ent or ent.get("source_hash") != source_hash():
+        return None
+    return ent.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.out = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=self.out, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.out.flush()
+        with open(self.out.name) as f:
+            rows = [r.strip().split(", ") for r in f if r.strip()]
+        os.unlink(self.out.name)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            if len(r) < 9:
+                continue
+            try:
+                sm.append(float(r[1]))
+                smax.append(float(r[2]))
+            except ValueError:
+                continue
+            for name, v in zip(names, r[5:9]):
+                if v.strip().lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def make_inputs(cfg: int, batch: int):
+    if cfg == 4:
+        w = workloads.config(4, batch=batch)
+    else:
+        w = workloads.config(cfg, batch=batch)
+    return w
+
+
+# --------------------------------------------------------------------- ours
+
+def run_ours(args, rank: int, world: int, local_rank: int):
+    import torch
+    from paper_2608_08340_gb300.index import Index
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    cfg = args.config
+    batch = args.batch or default_batch(cfg)
+    w = make_inputs(cfg, batch)
+
+    def to_dev(a):
+        if a.dtype == np.uint16:
+            return torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).to(dev)
+        return torch.from_numpy(a).to(dev)
+
+    def to_pinned(a):
+        t = (torch.from_numpy(a.view(np.int16)).view(torch.bfloat16) if a.dtype == np.uint16
+             else torch.from_numpy(a))
+        return t.pin_memory()
+
+    idx = Index(to_dev(w.E_data))
+    if cfg == 3:
+        idx.set_sparse(w.doc_indptr, w.doc_terms, w.vocab, w.k1, w.b)
+        q_indptr = torch.from_numpy(w.q_indptr).to(dev)
+        q_terms = torch.from_numpy(w.q_terms).to(dev)
+    idx.reserve(w.q, w.k)
+    idx.enable_timing(True)
+    Q = to_dev(w.Q_data)
+    Qh = to_pinned(w.Q_data)
+    ids = torch.empty((w.q, w.k), dtype=torch.int64, device=dev)
+    scores = torch.empty((w.q, w.k), dtype=torch.float32, device=dev)
+    ids_h = torch.empty((w.q, w.k), dtype=torch.int64).pin_memory()
+    scores_h = torch.empty((w.q, w.k), dtype=torch.float32).pin_memory()
+    ups = []
+    if cfg == 4:
+        for r in range(4):
+            u_ids, u_rows = workloads.upsert_batch(w.n, w.d, 4096, r + 1, w.dtype)
+            ups.append((u_ids, to_dev(u_rows), to_pinned(u_rows)))
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step(i, host=False):
+        if cfg == 4:
+            u_ids, u_dev, u_host = ups[i % len(ups)]
+            idx.upsert(u_ids, u_host if host else u_dev)
+        if host:
+            if cfg == 3:
+                raise RuntimeError("unreachable")
+            idx.search_host(Qh, w.k, out=(ids_h, scores_h))
+        elif cfg == 3:
+            idx.hybrid_search(Q, q_indptr, q_terms, w.alpha, w.k)
+        else:
+            idx.search(Q, w.k, out=(ids, scores))
+
+    launches_per_step = 2 + (1 if cfg in (3, 4) else 0)
+
+    for i in range(args.warmup):
+        flush.zero_()
+        step(i)
+    torch.cuda.synchronize()
+    idx.check()
+
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    step_ms, search_ms, lex_ms, merge_ms = [], [], [], []
+    with ClockSampler(local_rank) as clocks:
+        for i in range(args.steps):
+            flush.zero_()
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            step(i)
+            b.record(stream)
+            t = idx.last_timing()          # waits for this step
+            step_ms.append(a.elapsed_time(b))
+            search_ms.append(t["search_ms"])
+            merge_ms.append(t["merge_ms"])
+            lex_ms.append(t["lexical_ms"])
+        torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    idx.check()
+
+    # end to end: host queries in, host results out, through the C ABI
+    e2e_ms = []
+    if cfg != 3:
+        for i in range(args.warmup):
+            step(i, host=True)
+        for i in range(args.steps):
+            flush.zero_()
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            step(i, host=True)                 # synchronous call
+            e2e_ms.append((time.perf_counter() - t0) * 1e3)
+    else:
+        # hybrid: copy queries and terms in, read results out, around the call
+        for i in range(args.steps + args.warmup):
+            flush.zero_()
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            Qd = Qh.to(dev, non_blocking=True)
+            qi = torch.from_numpy(w.q_indptr).to(dev, non_blocking=True)
+            qt = torch.from_numpy(w.q_terms).to(dev, non_blocking=True)
+            r_ids, r_sc = idx.hybrid_search(Qd, qi, qt, w.alpha, w.k)
+            ids_h.copy_(r_ids)
+            scores_h.copy_(r_sc)
+            torch.cuda.synchronize()
+            if i >= args.warmup:
+                e2e_ms.append((time.perf_counter() - t0) * 1e3)
+
+    total_ms = sum(step_ms)
+    e2e_total = sum(e2e_ms)
+    if world > 1:
+        tt = torch.tensor([total_ms, e2e_total], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        total_ms, e2e_total = float(tt[0]), float(tt[1])
+    if rank != 0:
+        return None
+
+    nbytes, flops = roofline_terms(w, cfg)
+    hbm, tflops, peak_src = peaks()
+    t_kernel = statistics.mean(search_ms) * 1e-3
+    t_bytes = nbytes / (hbm * 1e9)
+    t_flops = flops / (tflops * 1e12)
+    elem_bf16 = w.dtype == "bf16"
+    if t_flops > t_bytes and elem_bf16:
+        roof = {"bound": "tensor", "achieved": flops / t_kernel / 1e12, "peak": tflops,
+                "unit": "TFLOP/s"}
+    else:
+        roof = {"bound": "hbm", "achieved": nbytes / t_kernel / 1e9, "peak": hbm, "unit": "GB/s"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    roof["peak_source"] = f"{peak_src} (MEASURED_PEAKS.json)" if peak_src == "measured" else peak_src
+    roof["kernel"] = "tc_search_kernel" if idx.last_path == "tc" else "simt_search_kernel"
+    roof["kernel_ms_mean"] = statistics.mean(search_ms)
+    roof["merge_ms_mean"] = statistics.mean(merge_ms)
+    if cfg == 3:
+        roof["bm25_ms_mean"] = statistics.mean(lex_ms)
+    roof["algorithmic_bytes"] = nbytes
+    roof["algorithmic_flops"] = flops
+    roof["roofline_time_frac"] = max(t_bytes, t_flops) / (statistics.mean(step_ms) * 1e-3)
+    key = f"cfg{cfg}_q{w.q}"
+    roof["traffic"] = ncu_traffic(key)
+
+    queries_all = w.q * args.steps * world
+    value = queries_all / (total_ms * 1e-3)
+    h2d = w.q * w.d * (2 if elem_bf16 else 4)
+    if cfg == 4:
+        h2d += 4096 * (w.d * 2 + 8)
+    if cfg == 3:
+        h2d += w.q_indptr.nbytes + w.q_terms.nbytes
+    d2h = w.q * w.k * 12
+    result = {
+        "metric": f"queries/s at top-{w.k}", "value": value, "unit": "queries/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
+        "config": {"workload": workload_name(cfg, w), "config_index": cfg, "n": w.n, "d": w.d,
+                   "q": w.q, "k": w.k, "parallelism": f"replicas{world}",
+                   "l2": f"flushed before every step ({L2_FLUSH_BYTES >> 20} MiB write)"},
+        "roofline": roof,
+        "e2e": {"value": queries_all / (e2e_total * 1e-3), "unit": "queries/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "api": "oprag_search_host" if cfg != 3 else "oprag_hybrid_search + torch copies"},
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clocks.summary(),
+        "path": idx.last_path,
+    }
+    idx.close()
+    return result, w
+
+
+# --------------------------------------------------------------------- oracle
+
+def oracle_queries_per_s(w, cfg, nq: int, threads: int, offset: int = 0):
+    import oracle
+    rows = (np.arange(nq) + offset) % w.q
+    Qs = w.Q_data[rows]
+    t0 = time.perf_counter()
+    if cfg == 3:
+        qts = [w.q_terms[w.q_indptr[r]:w.q_indptr[r + 1]] for r in rows]
+        qip = np.zeros(nq + 1, np.int32)
+        qip[1:] = np.cumsum([len(t) for t in qts])
+        oracle.hybrid_search(w.E_data, Qs, w.doc_indptr, w.doc_terms, w.vocab, qip,
+                             np.concatenate(qts).astype(np.int32), w.alpha, w.k, w.k1, w.b,
+                             nthreads=threads)
+    else:
+        oracle.search(w.E_data, Qs, w.k, nthreads=threads)
+    return nq / (time.perf_counter() - t0)
+
+
+def cpu_baseline(w, cfg, budget_s: float = 12.0):
+    """The oracle as it stands, on all host cores, on a bounded sample sized
+    from a short pilot to about budget_s seconds."""
+    threads = os.cpu_count() or 1
+    pilot = max(threads, 8)
+    rate = oracle_queries_per_s(w, cfg, pilot, threads)
+    nq = int(min(max(pilot, rate * budget_s), 4 * w.q))
+    nq = max(threads, nq // threads * threads)
+    rate = oracle_queries_per_s(w, cfg, nq, threads, offset=pilot)
+    return {"value": rate, "unit": "queries/s", "cores": threads, "kind": "oracle",
+            "sample": f"{nq} queries of the same workload (rows taken cyclically), full "
+                      f"fp64 scoring + full sort per query, {threads} threads"}
+
+
+def run_reference(args):
+    cfg = args.config
+    batch = args.batch or default_batch(cfg)
+    w = make_inputs(cfg, batch)
+    threads = os.cpu_count() or 1
+    # each step: a bounded sample of the step's queries (whole run within minutes)
+    pilot = oracle_queries_per_s(w, cfg, max(threads, 8), threads)
+    per_step = int(max(threads, min(w.q, pilot * 4.0)))
+    times, done = [], 0
+    for i in range(args.warmup):
+        oracle_queries_per_s(w, cfg, threads, threads)
+    for i in range(args.steps):
+        t0 = time.perf_counter()
+        oracle_queries_per_s(w, cfg, per_step, threads, offset=i * per_step)
+        times.append(time.perf_counter() - t0)
+        done += per_step
+    value = done / sum(times)
+    out = {
+        "impl": "reference", "metric": f"queries/s at top-{w.k}", "value": value,
+        "unit": "queries/s", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * sum(times) / len(times), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": workload_name(cfg, w), "config_index": cfg, "n": w.n, "d": w.d,
+                   "q": w.q, "k": w.k, "parallelism": "host threads"},
+        "cpu_baseline": {"value": value, "unit": "queries/s", "cores": threads,
+                         "kind": "oracle",
+                         "sample": f"{per_step} queries per step of the {w.q}-query batch"},
+        "e2e": {"value": value, "unit": "queries/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(out))
+
+
+def main():
+    args = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        if rank == 0:
+            run_reference(args)
+        return
+    if world > 1:
+        import torch
+        torch.cuda.set_device(local_rank)
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    res = run_ours(args, rank, world, local_rank)
+    if world > 1:
+        import torch
+        torch.distributed.destroy_process_group()
+    if res is None:
+        return
+    result, w = res
+    if not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline(w, args.config)
+    print(json.dumps(result))
+
+
+if __name__ == "__main__":
+    main()

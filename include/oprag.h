@@ -1,0 +1,206 @@
+/*
+ * oprag.h -- C ABI of the GB300 retrieval hot path of OpRAG (arxiv 2608.08340).
+ *
+ * The library implements, on one GPU, the data-parallel core of the paper's
+ * retrieval operator:
+ *   - exact top-k inner-product search of a query batch against a chunk
+ *     embedding index (Op_retrieve, Sec. 3.2: R_k = Op_retrieve(q, I), and the
+ *     TopK display of Sec. 4.4);
+ *   - hybrid dense + BM25 search with the weighted score fusion of Sec. 4.4;
+ *   - in-place index upsert (Op_upsert, Sec. 3.2: I' = Op_upsert(I, E; b_u)).
+ *
+ * Conventions for every function below
+ *   - Return value: OPRAG_OK (0) or a negative OPRAG_ERR_* code; the message
+ *     of the last failure on the calling thread is oprag_last_error().  A
+ *     failing call writes nothing to its outputs and leaves the index as it
+ *     was, unless the code is OPRAG_ERR_CUDA.
+ *   - "device" pointers are CUDA device memory of the GPU that was current when
+ *     the index was created; "host" pointers are ordinary (pageable or pinned)
+ *     host memory.  The caller keeps ownership of everything it passes in.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
+ *     stream).  Asynchronous calls only enqueue work on it.  Calls on one index
+ *     share its scratch memory: the library orders each call after the previous
+ *     call on the same index (cross-stream calls wait on an event), but one
+ *     index must not be used from two host threads at once.
+ *   - Ranking: score descending, equal scores broken by the lower chunk id.
+ *   - dtype codes: OPRAG_F32 (IEEE binary32) or OPRAG_BF16 (bfloat16, stored as
+ *     the upper 16 bits of a binary32).
+ *   - Inputs are finite.  Vectors are used as given: the index never
+ *     normalises (normalisation belongs to embedding, Sec. 4.3).
+ */
+#ifndef OPRAG_H
+#define OPRAG_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define OPRAG_API __attribute__((visibility("default")))
+#else
+#define OPRAG_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define OPRAG_F32 0
+#define OPRAG_BF16 1
+
+#define OPRAG_OK 0
+#define OPRAG_ERR_INVALID_ARG (-1) /* null pointer, bad size, k out of range, dtype mismatch */
+#define OPRAG_ERR_RANGE (-2)       /* an upsert id outside [0, n) */
+#define OPRAG_ERR_OOM (-3)         /* device or host allocation failed */
+#define OPRAG_ERR_CUDA (-4)        /* a CUDA call or an earlier asynchronous launch failed */
+#define OPRAG_ERR_NOT_READY (-5)   /* hybrid search before oprag_index_set_sparse */
+#define OPRAG_ERR_DEVICE (-6)      /* a kernel gave up waiting (bounded wait expired) */
+
+/* Largest k accepted by the search calls. */
+#define OPRAG_K_MAX 256
+
+typedef struct oprag_index oprag_index;
+
+/*
+ * Creates an index of n chunk embeddings of dimension d, stored on the current
+ * GPU as dtype (OPRAG_F32 or OPRAG_BF16) in row-major n x d layout (the
+ * "contiguous" vector buffer of Sec. 4.2).
+ *   emb        n x d row-major, element type src_dtype; host memory if
+ *              emb_on_device == 0, else device memory.  Copied; not retained.
+ *   src_dtype  OPRAG_F32 or OPRAG_BF16.  F32 input into a BF16 index is
+ *              rounded to nearest even; BF16 input into an F32 index is refused.
+ *   d          1..8192, a multiple of 8.
+ *   n          1 .. 2^31 - 1.
+ * Synchronous.  *out receives the handle (NULL on failure).
+ */
+OPRAG_API int oprag_index_create(oprag_index **out, const void *emb, int64_t n, int32_t d, int32_t dtype,
+                       int32_t src_dtype, int32_t emb_on_device);
+
+/* Frees the index and all its device memory after its pending work is done.
+ * NULL is allowed. */
+OPRAG_API void oprag_index_destroy(oprag_index *idx);
+
+/* Shape of the index: any out-pointer may be NULL. */
+OPRAG_API int oprag_index_info(const oprag_index *idx, int64_t *n, int32_t *d, int32_t *dtype,
+                     int32_t *device);
+
+/* Device pointer of the n x d embedding matrix (read-only use; valid until
+ * destroy).  For tests and zero-copy readers. */
+OPRAG_API const void *oprag_index_data(const oprag_index *idx);
+
+/*
+ * Copies rows [first, first + count) of the index into host memory `out`
+ * (count x d elements of the index dtype).  Synchronous.  For tests.
+ */
+OPRAG_API int oprag_index_get_rows(const oprag_index *idx, int64_t first, int64_t count, void *out);
+
+/*
+ * Pre-allocates the scratch memory that searches of up to q_max queries and
+ * k_max results need, so that later calls allocate nothing.  Optional: search
+ * calls grow the scratch on demand (which synchronises the device once).
+ */
+OPRAG_API int oprag_index_reserve(oprag_index *idx, int32_t q_max, int32_t k_max);
+
+/*
+ * Upsert (Sec. 3.2 Op_upsert; Sec. 4.1: updates are coalesced and committed in
+ * bulk).  Row i of `rows` overwrites chunk ids[i]; when an id repeats, the
+ * later entry wins.
+ *   ids              host, m int64 chunk ids in [0, n); validated before any
+ *                    write (OPRAG_ERR_RANGE, nothing written).
+ *   rows             m x d row-major of rows_dtype; device memory if
+ *                    rows_on_device, else host memory (copied before return).
+ *   rows_dtype       as for create: F32 rows into a BF16 index are rounded to
+ *                    nearest even.
+ * Asynchronous on `stream`; later searches on the same index see the new rows.
+ */
+OPRAG_API int oprag_upsert(oprag_index *idx, const int64_t *ids, const void *rows, int64_t m,
+                 int32_t rows_dtype, int32_t rows_on_device, void *stream);
+
+/*
+ * Exact dense top-k search (Sec. 3.2 Op_retrieve; Sec. 4.4 dense scores by
+ * matrix operations and partial top-k selection).  For each query i:
+ * out[i][0..k) = the k chunks with the largest inner product <Q_i, E_c>.
+ *   queries      device, q x d row-major, the index dtype, 16-byte aligned.
+ *   q            >= 0 (0 is a no-op).
+ *   k            1 .. min(n, OPRAG_K_MAX).
+ *   out_ids      device, q x k int64, row-major, best first.
+ *   out_scores   device, q x k float: the scores, accumulated in fp32.
+ * Asynchronous on `stream`.
+ */
+OPRAG_API int oprag_search(oprag_index *idx, const void *queries, int32_t q, int32_t k, int64_t *out_ids,
+                 float *out_scores, void *stream);
+
+/*
+ * Same search with host buffers: copies the q x d queries from host memory,
+ * searches and copies ids and scores back to host memory.  Synchronous; also
+ * reports a device-side wait failure of this call (OPRAG_ERR_DEVICE).
+ */
+OPRAG_API int oprag_search_host(oprag_index *idx, const void *queries, int32_t q, int32_t k,
+                      int64_t *out_ids, float *out_scores, void *stream);
+
+/*
+ * Attaches the lexical side used by the hybrid search: the bag of term ids of
+ * every chunk, as CSR on the host (doc_indptr[n + 1], doc_terms[doc_indptr[n]],
+ * term ids in [0, vocab)).  BM25 statistics (document frequency, average
+ * length, per-posting weights) are built here, in fp64 on the host, with the
+ * Okapi form and idf(t) = ln(1 + (N - df + 0.5) / (df + 0.5)).  Synchronous;
+ * replaces a previous sparse side.
+ */
+OPRAG_API int oprag_index_set_sparse(oprag_index *idx, const int32_t *doc_indptr, const int32_t *doc_terms,
+                           int32_t vocab, float k1, float b);
+
+/*
+ * Hybrid search with the weighted score fusion of Sec. 4.4:
+ *   score(d, q) = alpha * <q, e_d> + (1 - alpha) * BM25(q, d) / max_d' BM25(q, d'),
+ * with the lexical part 0 for a query whose maximum BM25 is 0, followed by the
+ * same top-k as oprag_search.
+ *   queries      device, q x d (index dtype), 16-byte aligned.
+ *   q_indptr     device, q + 1 int32 offsets into q_terms.
+ *   q_terms      device, int32 term ids (repeats count again; ids outside
+ *                [0, vocab) contribute nothing).
+ *   alpha        dense weight w_d; the lexical weight is w_l = 1 - alpha.
+ * Asynchronous on `stream`.  OPRAG_ERR_NOT_READY without a sparse side.
+ */
+OPRAG_API int oprag_hybrid_search(oprag_index *idx, const void *queries, int32_t q, const int32_t *q_indptr,
+                        const int32_t *q_terms, float alpha, int32_t k, int64_t *out_ids,
+                        float *out_scores, void *stream);
+
+/*
+ * Waits for the index's pending work and reports whether a kernel of it gave
+ * up a bounded wait since the last check (OPRAG_ERR_DEVICE; the flag is then
+ * cleared) or a CUDA error occurred (OPRAG_ERR_CUDA).
+ */
+OPRAG_API int oprag_index_check(oprag_index *idx);
+
+/* Test hooks: 0 = automatic choice.  OPRAG_OPT_PATH: 1 forces the SIMT
+ * streaming kernel, 2 the tensor-core kernel (bf16 only).  OPRAG_OPT_BLOCK_N:
+ * corpus rows per tensor-core tile (64 or 256). */
+#define OPRAG_OPT_PATH 1
+#define OPRAG_OPT_BLOCK_N 2
+OPRAG_API int oprag_index_set_option(oprag_index *idx, int32_t option, int32_t value);
+
+/* OPRAG_OPT_TIMING: 1 makes every later search record CUDA events, on the
+ * call's stream, around its lexical (BM25) kernel, its main search kernel and
+ * its merge kernel; oprag_index_last_timing() reads them.  0 (default) off. */
+#define OPRAG_OPT_TIMING 3
+
+/*
+ * Device durations (milliseconds) of the kernels of the last search issued
+ * with timing on: lexical_ms (BM25 pass of a hybrid search, 0 for a dense
+ * search), search_ms (score contraction + fused selection), merge_ms (final
+ * top-k reduction).  Waits for that search to finish.  Any out-pointer may be
+ * NULL.  OPRAG_ERR_NOT_READY if no timed search was issued.
+ */
+OPRAG_API int oprag_index_last_timing(oprag_index *idx, float *lexical_ms, float *search_ms,
+                                      float *merge_ms);
+
+/* Which kernel family served the last search on this index: 1 SIMT, 2 tensor
+ * core, 0 none yet. */
+OPRAG_API int oprag_index_last_path(const oprag_index *idx);
+
+/* Message of the last failed call on this thread ("" if none). */
+OPRAG_API const char *oprag_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* OPRAG_H */

@@ -1,0 +1,89 @@
+// Internal host-side interface between the C-ABI layer (oprag.cu) and the
+// kernel translation units.  Not part of the public header.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace oprag {
+
+enum Dtype : int { kF32 = 0, kBF16 = 1 };
+
+// Kept-list length used for a requested k: 8 or 32 (register lists), 128 or
+// 256 (buffered lists).
+inline int list_len_for(int k) { return k <= 8 ? 8 : k <= 32 ? 32 : k <= 128 ? 128 : 256; }
+
+// Partial top-K lists written by a search kernel and read by the merge.  The
+// list of query row `row` of query tile `tile` produced by producer `p` starts
+// at keys + ((tile * P + p) * TH + row) * stride and is sorted best first.
+struct ListSet {
+  const uint64_t* keys;
+  int P;
+  int TH;
+  int stride;
+};
+
+// Optional lexical part of the fused score (Sec. 4.4 weighted fusion):
+// f = alpha * dense + (1 - alpha) * bm25[q][id] / max_q, zero lexical part when
+// max_q <= 0.  bm25 == nullptr means a plain dense search.
+struct Fusion {
+  const float* bm25;      // q x ld, row-major
+  int64_t ld;
+  const float* bm25_max;  // q
+  float alpha;
+};
+
+struct SearchShape {
+  int64_t n;
+  int d;
+  int q;
+  int k;
+};
+
+// --- SIMT streaming search (fp32 or bf16; any q, meant for small q).
+size_t simt_scratch_bytes(int dtype, const SearchShape& s, int grid);
+int simt_grid(const SearchShape& s, int num_sms);
+cudaError_t launch_simt_search(int dtype, const void* E, const void* Q, const SearchShape& s,
+                               const Fusion& fu, void* scratch, int grid, ListSet* lists,
+                               cudaStream_t st);
+
+// --- tcgen05 tensor-core search (bf16).
+struct TcPlan {
+  int block_n;     // corpus rows per tile: 64, 128 or 256
+  int grid;        // CTAs (persistent)
+  int qt;          // query tiles of 128
+  int slots;       // query tiles visited per CTA
+  int P;           // lists per query tile
+  int stages;
+  size_t smem;
+};
+TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n);
+size_t tc_scratch_bytes(const SearchShape& s, const TcPlan& p);
+cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s, const Fusion& fu,
+                             const TcPlan& plan, void* scratch, int* dev_err, ListSet* lists,
+                             cudaStream_t st);
+
+// --- final merge of partial lists into the sorted top-k per query.
+cudaError_t launch_merge(const ListSet& ls, int q, int k, int64_t* out_ids, float* out_scores,
+                         cudaStream_t st);
+
+// --- BM25 matrix pass (lexical part of the hybrid search).
+struct SparseIndex {
+  int vocab;
+  int64_t nnz;               // postings
+  const int64_t* post_ptr;   // device, vocab + 1
+  const int32_t* post_doc;   // device, nnz, ascending per term
+  const float* post_w;       // device, nnz: idf * tf (k1+1) / (tf + k1 (1 - b + b |d| / avgdl))
+};
+cudaError_t launch_bm25_matrix(const SparseIndex& sp, int64_t n, const int32_t* q_indptr,
+                               const int32_t* q_terms, int q, float* out, int64_t ld,
+                               float* out_max, cudaStream_t st);
+
+// --- upsert / conversion.
+cudaError_t launch_scatter_rows(int index_dtype, void* E, int d, const void* rows, int rows_dtype,
+                                const int64_t* src_dst /* pairs: source row, destination row */,
+                                int64_t count, cudaStream_t st);
+cudaError_t launch_convert_f32_bf16(const float* src, void* dst, int64_t count, cudaStream_t st);
+
+}  // namespace oprag

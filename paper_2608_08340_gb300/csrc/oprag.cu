@@ -1,0 +1,638 @@
+// Host side of the C ABI declared in include/oprag.h: the index object,
+// argument checking, scratch management and the choice of kernel family.
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <unordered_set>
+#include <vector>
+
+#include "../../include/oprag.h"
+#include "internal.h"
+
+using namespace oprag;
+
+namespace {
+
+thread_local std::string g_err;
+
+int fail(int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_err = buf;
+  return code;
+}
+
+int cuda_fail(cudaError_t e, const char* what) {
+  return fail(OPRAG_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+int ok() {
+  g_err.clear();
+  return OPRAG_OK;
+}
+
+size_t elem_size(int dtype) { return dtype == OPRAG_F32 ? 4 : 2; }
+
+// Makes the index's device current for the duration of a call.
+struct DeviceGuard {
+  int prev = -1;
+  bool changed = false;
+  explicit DeviceGuard(int dev) {
+    if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) {
+      changed = cudaSetDevice(dev) == cudaSuccess;
+    }
+  }
+  ~DeviceGuard() {
+    if (changed) cudaSetDevice(prev);
+  }
+};
+
+// bf16 queries with at most this many rows take the SIMT stream by default.
+constexpr int kSimtMaxQueriesBf16 = 4;
+// Largest BM25 matrix block (floats) materialised per hybrid pass.
+constexpr int64_t kLexMaxElems = int64_t(1) << 28;
+
+}  // namespace
+
+struct oprag_index {
+  int device = 0;
+  int num_sms = 1;
+  int64_t n = 0;
+  int d = 0;
+  int dtype = OPRAG_BF16;
+  void* emb = nullptr;
+  int* dev_err = nullptr;
+  cudaEvent_t done = nullptr;
+
+  void* scratch = nullptr;     // partial top-k lists
+  size_t scratch_bytes = 0;
+  float* lex = nullptr;        // BM25 block (q x ld) followed by q maxima
+  size_t lex_bytes = 0;
+  void* stage = nullptr;       // upsert staging / host-buffer search staging
+  size_t stage_bytes = 0;
+
+  bool has_sparse = false;
+  int vocab = 0;
+  int64_t nnz = 0;
+  int64_t* post_ptr = nullptr;
+  int32_t* post_doc = nullptr;
+  float* post_w = nullptr;
+
+  int opt_path = 0;
+  int opt_block_n = 0;
+  int last_path = 0;
+
+  // Optional kernel timing: events before the lexical pass, before the
+  // search kernel, before the merge kernel and after it.
+  bool timing = false;
+  bool timed = false;      // the last search recorded its events
+  bool timed_lex = false;  // ... including a lexical pass
+  cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
+
+  // Waits until all work enqueued on this index is done.
+  cudaError_t drain() { return done ? cudaEventSynchronize(done) : cudaSuccess; }
+
+  // Grows a device buffer.  The old buffer may still be read by work this or
+  // an earlier call enqueued, so the whole device is drained first.
+  int ensure(void** buf, size_t* cur, size_t need, const char* what) {
+    if (need <= *cur) return OPRAG_OK;
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(e, "waiting for pending work");
+    if (*buf) cudaFree(*buf);
+    *buf = nullptr;
+    *cur = 0;
+    const size_t want = need + need / 4;
+    if (cudaMalloc(buf, want) != cudaSuccess) {
+      cudaGetLastError();
+      *buf = nullptr;
+      return fail(OPRAG_ERR_OOM, "cannot allocate %zu bytes of %s", want, what);
+    }
+    *cur = want;
+    return OPRAG_OK;
+  }
+
+  void free_sparse() {
+    if (post_ptr) cudaFree(post_ptr);
+    if (post_doc) cudaFree(post_doc);
+    if (post_w) cudaFree(post_w);
+    post_ptr = nullptr;
+    post_doc = nullptr;
+    post_w = nullptr;
+    has_sparse = false;
+  }
+};
+
+namespace {
+
+int begin_call(oprag_index* idx, cudaStream_t st) {
+  cudaGetLastError();  // clear a stale, non-sticky error of another library
+  cudaError_t e = cudaStreamWaitEvent(st, idx->done, 0);
+  if (e != cudaSuccess) return cuda_fail(e, "ordering after the previous call");
+  return OPRAG_OK;
+}
+
+int end_call(oprag_index* idx, cudaStream_t st) {
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "kernel launch");
+  e = cudaEventRecord(idx->done, st);
+  if (e != cudaSuccess) return cuda_fail(e, "recording completion");
+  return ok();
+}
+
+int choose_path(const oprag_index* idx, int q) {
+  if (idx->dtype == OPRAG_F32) return 1;
+  if (idx->opt_path == 1 || idx->opt_path == 2) return idx->opt_path;
+  return q <= kSimtMaxQueriesBf16 ? 1 : 2;
+}
+
+// Dense (or fused) top-k of q queries; all pointers on the device.
+int run_search(oprag_index* idx, const void* Q, int q, int k, const Fusion& fu, int64_t* out_ids,
+               float* out_scores, cudaStream_t st) {
+  SearchShape s{idx->n, idx->d, q, k};
+  const int path = choose_path(idx, q);
+  ListSet lists{};
+  cudaError_t e;
+  if (path == 1) {
+    const int grid = simt_grid(s, idx->num_sms);
+    int rc = idx->ensure(&idx->scratch, &idx->scratch_bytes, simt_scratch_bytes(idx->dtype, s, grid),
+                         "search scratch");
+    if (rc) return rc;
+    if (idx->timing) cudaEventRecord(idx->ev[1], st);
+    e = launch_simt_search(idx->dtype, idx->emb, Q, s, fu, idx->scratch, grid, &lists, st);
+  } else {
+    const TcPlan plan = tc_plan(s, idx->num_sms, idx->opt_block_n);
+    int rc = idx->ensure(&idx->scratch, &idx->scratch_bytes, tc_scratch_bytes(s, plan),
+                         "search scratch");
+    if (rc) return rc;
+    if (idx->timing) cudaEventRecord(idx->ev[1], st);
+    e = launch_tc_search(idx->emb, Q, s, fu, plan, idx->scratch, idx->dev_err, &lists, st);
+  }
+  if (e != cudaSuccess) return cuda_fail(e, "search kernel");
+  if (idx->timing) cudaEventRecord(idx->ev[2], st);
+  e = launch_merge(lists, q, k, out_ids, out_scores, st);
+  if (e != cudaSuccess) return cuda_fail(e, "merge kernel");
+  if (idx->timing) cudaEventRecord(idx->ev[3], st);
+  idx->timed = idx->timing;
+  idx->last_path = path;
+  return OPRAG_OK;
+}
+
+int check_search_args(const oprag_index* idx, const void* queries, int q, int k,
+                      const void* out_ids, const void* out_scores) {
+  if (!idx) return fail(OPRAG_ERR_INVALID_ARG, "index is NULL");
+  if (q < 0) return fail(OPRAG_ERR_INVALID_ARG, "q = %d < 0", q);
+  if (k < 1 || k > OPRAG_K_MAX || k > idx->n)
+    return fail(OPRAG_ERR_INVALID_ARG, "k = %d outside [1, min(n = %lld, %d)]", k,
+                static_cast<long long>(idx->n), OPRAG_K_MAX);
+  if (q > 0 && (!queries || !out_ids || !out_scores))
+    return fail(OPRAG_ERR_INVALID_ARG, "NULL queries or output buffer");
+  if (q > 0 && (reinterpret_cast<uintptr_t>(queries) & 15))
+    return fail(OPRAG_ERR_INVALID_ARG, "queries must be 16-byte aligned");
+  return OPRAG_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* oprag_last_error(void) { return g_err.c_str(); }
+
+int oprag_index_create(oprag_index** out, const void* emb, int64_t n, int32_t d, int32_t dtype,
+                       int32_t src_dtype, int32_t emb_on_device) {
+  if (!out) return fail(OPRAG_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  if (!emb) return fail(OPRAG_ERR_INVALID_ARG, "emb is NULL");
+  if (n < 1 || n > 0x7FFFFFFFLL) return fail(OPRAG_ERR_INVALID_ARG, "n = %lld out of range", (long long)n);
+  if (d < 1 || d > 8192 || d % 8)
+    return fail(OPRAG_ERR_INVALID_ARG, "d = %d must be a multiple of 8 in [8, 8192]", d);
+  if ((dtype != OPRAG_F32 && dtype != OPRAG_BF16) || (src_dtype != OPRAG_F32 && src_dtype != OPRAG_BF16))
+    return fail(OPRAG_ERR_INVALID_ARG, "unknown dtype");
+  if (dtype == OPRAG_F32 && src_dtype == OPRAG_BF16)
+    return fail(OPRAG_ERR_INVALID_ARG, "bf16 input into an f32 index is not supported");
+
+  oprag_index* idx = new (std::nothrow) oprag_index();
+  if (!idx) return fail(OPRAG_ERR_OOM, "host allocation");
+  cudaGetLastError();
+  cudaError_t e = cudaGetDevice(&idx->device);
+  if (e != cudaSuccess) {
+    delete idx;
+    return cuda_fail(e, "no CUDA device");
+  }
+  cudaDeviceGetAttribute(&idx->num_sms, cudaDevAttrMultiProcessorCount, idx->device);
+  idx->n = n;
+  idx->d = d;
+  idx->dtype = dtype;
+  const size_t count = static_cast<size_t>(n) * d;
+  const size_t bytes = count * elem_size(dtype);
+  auto bail = [&](int rc) {
+    oprag_index_destroy(idx);
+    return rc;
+  };
+  if (cudaMalloc(&idx->emb, bytes) != cudaSuccess) {
+    cudaGetLastError();
+    idx->emb = nullptr;
+    return bail(fail(OPRAG_ERR_OOM, "cannot allocate %zu bytes for the index", bytes));
+  }
+  if (cudaMalloc(reinterpret_cast<void**>(&idx->dev_err), sizeof(int)) != cudaSuccess) {
+    cudaGetLastError();
+    idx->dev_err = nullptr;
+    return bail(fail(OPRAG_ERR_OOM, "cannot allocate the error word"));
+  }
+  if ((e = cudaEventCreateWithFlags(&idx->done, cudaEventDisableTiming)) != cudaSuccess)
+    return bail(cuda_fail(e, "event"));
+  cudaStream_t st;
+  if ((e = cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking)) != cudaSuccess)
+    return bail(cuda_fail(e, "stream"));
+  e = cudaMemsetAsync(idx->dev_err, 0, sizeof(int), st);
+  if (e == cudaSuccess) {
+    if (src_dtype == dtype) {
+      e = cudaMemcpyAsync(idx->emb, emb, bytes, emb_on_device ? cudaMemcpyDeviceToDevice
+                                                              : cudaMemcpyHostToDevice, st);
+    } else if (emb_on_device) {
+      e = launch_convert_f32_bf16(static_cast<const float*>(emb), idx->emb, count, st);
+    } else {
+      // Host fp32 -> device staging in slices -> bf16 rounding kernel.
+      const size_t slice = std::min<size_t>(count, size_t(1) << 26);
+      float* tmp = nullptr;
+      e = cudaMalloc(&tmp, slice * sizeof(float));
+      for (size_t off = 0; e == cudaSuccess && off < count; off += slice) {
+        const size_t c = std::min(slice, count - off);
+        e = cudaMemcpyAsync(tmp, static_cast<const float*>(emb) + off, c * sizeof(float),
+                            cudaMemcpyHostToDevice, st);
+        if (e == cudaSuccess)
+          e = launch_convert_f32_bf16(tmp, static_cast<uint16_t*>(idx->emb) + off, c, st);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+      }
+      if (tmp) cudaFree(tmp);
+    }
+  }
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  cudaStreamDestroy(st);
+  if (e != cudaSuccess) return bail(cuda_fail(e, "copying the embeddings"));
+  if ((e = cudaEventRecord(idx->done, 0)) != cudaSuccess) return bail(cuda_fail(e, "event"));
+  *out = idx;
+  return ok();
+}
+
+void oprag_index_destroy(oprag_index* idx) {
+  if (!idx) return;
+  DeviceGuard g(idx->device);
+  idx->drain();
+  if (idx->emb) cudaFree(idx->emb);
+  if (idx->dev_err) cudaFree(idx->dev_err);
+  if (idx->scratch) cudaFree(idx->scratch);
+  if (idx->lex) cudaFree(idx->lex);
+  if (idx->stage) cudaFree(idx->stage);
+  idx->free_sparse();
+  if (idx->done) cudaEventDestroy(idx->done);
+  for (cudaEvent_t ev : idx->ev)
+    if (ev) cudaEventDestroy(ev);
+  delete idx;
+}
+
+int oprag_index_info(const oprag_index* idx, int64_t* n, int32_t* d, int32_t* dtype,
+                     int32_t* device) {
+  if (!idx) return fail(OPRAG_ERR_INVALID_ARG, "index is NULL");
+  if (n) *n = idx->n;
+  if (d) *d = idx->d;
+  if (dtype) *dtype = idx->dtype;
+  if (device) *device = idx->device;
+  return ok();
+}
+
+const void* oprag_index_data(const oprag_index* idx) { return idx ? idx->emb : nullptr; }
+
+int oprag_index_get_rows(const oprag_index* idx, int64_t first, int64_t count, void* out) {
+  if (!idx || !out) return fail(OPRAG_ERR_INVALID_ARG, "NULL argument");
+  if (first < 0 || count < 0 || first + count > idx->n)
+    return fail(OPRAG_ERR_RANGE, "rows [%lld, %lld) outside the index", (long long)first,
+                (long long)(first + count));
+  DeviceGuard g(idx->device);
+  const_cast<oprag_index*>(idx)->drain();
+  const size_t row = static_cast<size_t>(idx->d) * elem_size(idx->dtype);
+  cudaError_t e = cudaMemcpy(out, static_cast<const char*>(idx->emb) + first * row, count * row,
+                             cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "reading rows");
+  return ok();
+}
+
+int oprag_index_reserve(oprag_index* idx, int32_t q_max, int32_t k_max) {
+  if (!idx) return fail(OPRAG_ERR_INVALID_ARG, "index is NULL");
+  if (q_max < 1 || k_max < 1 || k_max > OPRAG_K_MAX)
+    return fail(OPRAG_ERR_INVALID_ARG, "bad reservation q_max=%d k_max=%d", q_max, k_max);
+  DeviceGuard g(idx->device);
+  SearchShape s{idx->n, idx->d, q_max, std::min<int>(k_max, static_cast<int>(std::min<int64_t>(idx->n, OPRAG_K_MAX)))};
+  size_t need = simt_scratch_bytes(idx->dtype, s, simt_grid(s, idx->num_sms));
+  if (idx->dtype == OPRAG_BF16) {
+    for (int bn : {64, 256}) {
+      for (int qq : {q_max, std::min(q_max, 128)}) {
+        SearchShape s2 = s;
+        s2.q = qq;
+        need = std::max(need, tc_scratch_bytes(s2, tc_plan(s2, idx->num_sms, bn)));
+      }
+    }
+  }
+  int rc = idx->ensure(&idx->scratch, &idx->scratch_bytes, need, "search scratch");
+  if (rc) return rc;
+  if (idx->has_sparse) {
+    const int64_t ld = (idx->n + 3) / 4 * 4;
+    const int64_t qc = std::min<int64_t>(q_max, std::max<int64_t>(1, kLexMaxElems / ld));
+    rc = idx->ensure(reinterpret_cast<void**>(&idx->lex), &idx->lex_bytes,
+                     sizeof(float) * static_cast<size_t>(qc * ld + qc), "BM25 block");
+    if (rc) return rc;
+  }
+  return ok();
+}
+
+int oprag_upsert(oprag_index* idx, const int64_t* ids, const void* rows, int64_t m,
+                 int32_t rows_dtype, int32_t rows_on_device, void* stream) {
+  if (!idx) return fail(OPRAG_ERR_INVALID_ARG, "index is NULL");
+  if (m < 0) return fail(OPRAG_ERR_INVALID_ARG, "m < 0");
+  if (m == 0) return ok();
+  if (!ids || !rows) return fail(OPRAG_ERR_INVALID_ARG, "NULL ids or rows");
+  if (rows_dtype != OPRAG_F32 && rows_dtype != OPRAG_BF16)
+    return fail(OPRAG_ERR_INVALID_ARG, "unknown rows dtype");
+  if (idx->dtype == OPRAG_F32 && rows_dtype == OPRAG_BF16)
+    return fail(OPRAG_ERR_INVALID_ARG, "bf16 rows into an f32 index are not supported");
+  for (int64_t i = 0; i < m; ++i)
+    if (ids[i] < 0 || ids[i] >= idx->n)
+      return fail(OPRAG_ERR_RANGE, "ids[%lld] = %lld outside [0, %lld)", (long long)i,
+                  (long long)ids[i], (long long)idx->n);
+  if (rows_on_device && (reinterpret_cast<uintptr_t>(rows) & 15))
+    return fail(OPRAG_ERR_INVALID_ARG, "device rows must be 16-byte aligned");
+  // The later entry of a repeated id wins: keep the last occurrence only.
+  std::vector<int64_t> pairs;
+  pairs.reserve(2 * m);
+  {
+    std::unordered_set<int64_t> seen;
+    seen.reserve(static_cast<size_t>(m) * 2);
+    for (int64_t i = m - 1; i >= 0; --i)
+      if (seen.insert(ids[i]).second) {
+        pairs.push_back(i);
+        pairs.push_back(ids[i]);
+      }
+  }
+  const int64_t count = static_cast<int64_t>(pairs.size() / 2);
+  DeviceGuard g(idx->device);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t row_bytes = static_cast<size_t>(idx->d) * elem_size(rows_dtype);
+  const size_t pair_bytes = pairs.size() * sizeof(int64_t);
+  const size_t pair_off = 0;
+  const size_t rows_off = (pair_bytes + 255) / 256 * 256;
+  const size_t need = rows_off + (rows_on_device ? 0 : static_cast<size_t>(m) * row_bytes);
+  int rc = idx->ensure(&idx->stage, &idx->stage_bytes, need, "upsert staging");
+  if (rc) return rc;
+  if ((rc = begin_call(idx, st))) return rc;
+  char* stage = static_cast<char*>(idx->stage);
+  cudaError_t e = cudaMemcpyAsync(stage + pair_off, pairs.data(), pair_bytes,
+                                  cudaMemcpyHostToDevice, st);
+  const void* src = rows;
+  if (e == cudaSuccess && !rows_on_device) {
+    e = cudaMemcpyAsync(stage + rows_off, rows, static_cast<size_t>(m) * row_bytes,
+                        cudaMemcpyHostToDevice, st);
+    src = stage + rows_off;
+  }
+  if (e != cudaSuccess) return cuda_fail(e, "copying the upsert batch");
+  e = launch_scatter_rows(idx->dtype, idx->emb, idx->d, src, rows_dtype,
+                          reinterpret_cast<const int64_t*>(stage + pair_off), count, st);
+  if (e != cudaSuccess) return cuda_fail(e, "upsert kernel");
+  return end_call(idx, st);
+}
+
+int oprag_search(oprag_index* idx, const void* queries, int32_t q, int32_t k, int64_t* out_ids,
+                 float* out_scores, void* stream) {
+  int rc = check_search_args(idx, queries, q, k, out_ids, out_scores);
+  if (rc) return rc;
+  if (q == 0) return ok();
+  DeviceGuard g(idx->device);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if ((rc = begin_call(idx, st))) return rc;
+  const Fusion none{nullptr, 0, nullptr, 0.f};
+  idx->timed_lex = false;
+  if ((rc = run_search(idx, queries, q, k, none, out_ids, out_scores, st))) return rc;
+  return end_call(idx, st);
+}
+
+int oprag_search_host(oprag_index* idx, const void* queries, int32_t q, int32_t k,
+                      int64_t* out_ids, float* out_scores, void* stream) {
+  int rc = check_search_args(idx, queries, q, k, out_ids, out_scores);
+  if (rc) return rc;
+  if (q == 0) return ok();
+  DeviceGuard g(idx->device);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t qbytes = static_cast<size_t>(q) * idx->d * elem_size(idx->dtype);
+  const size_t q_off = 0;
+  const size_t id_off = (qbytes + 255) / 256 * 256;
+  const size_t sc_off = id_off + (static_cast<size_t>(q) * k * sizeof(int64_t) + 255) / 256 * 256;
+  const size_t need = sc_off + static_cast<size_t>(q) * k * sizeof(float);
+  if ((rc = idx->ensure(&idx->stage, &idx->stage_bytes, need, "search staging"))) return rc;
+  if ((rc = begin_call(idx, st))) return rc;
+  char* stage = static_cast<char*>(idx->stage);
+  cudaError_t e = cudaMemcpyAsync(stage + q_off, queries, qbytes, cudaMemcpyHostToDevice, st);
+  if (e != cudaSuccess) return cuda_fail(e, "copying queries");
+  const Fusion none{nullptr, 0, nullptr, 0.f};
+  if ((rc = run_search(idx, stage + q_off, q, k, none, reinterpret_cast<int64_t*>(stage + id_off),
+                       reinterpret_cast<float*>(stage + sc_off), st)))
+    return rc;
+  e = cudaMemcpyAsync(out_ids, stage + id_off, static_cast<size_t>(q) * k * sizeof(int64_t),
+                      cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(out_scores, stage + sc_off, static_cast<size_t>(q) * k * sizeof(float),
+                        cudaMemcpyDeviceToHost, st);
+  if (e != cudaSuccess) return cuda_fail(e, "copying results");
+  if ((rc = end_call(idx, st))) return rc;
+  if ((e = cudaStreamSynchronize(st)) != cudaSuccess) return cuda_fail(e, "search");
+  return oprag_index_check(idx);
+}
+
+int oprag_index_set_sparse(oprag_index* idx, const int32_t* doc_indptr, const int32_t* doc_terms,
+                           int32_t vocab, float k1, float b) {
+  if (!idx || !doc_indptr) return fail(OPRAG_ERR_INVALID_ARG, "NULL argument");
+  if (vocab < 1) return fail(OPRAG_ERR_INVALID_ARG, "vocab = %d", vocab);
+  if (!(k1 >= 0.f) || !(b >= 0.f && b <= 1.f))
+    return fail(OPRAG_ERR_INVALID_ARG, "need k1 >= 0 and 0 <= b <= 1");
+  const int64_t n = idx->n;
+  if (doc_indptr[0] != 0) return fail(OPRAG_ERR_INVALID_ARG, "doc_indptr[0] != 0");
+  for (int64_t i = 0; i < n; ++i)
+    if (doc_indptr[i + 1] < doc_indptr[i])
+      return fail(OPRAG_ERR_INVALID_ARG, "doc_indptr decreases at %lld", (long long)i);
+  const int64_t total = doc_indptr[n];
+  if (total > 0 && !doc_terms) return fail(OPRAG_ERR_INVALID_ARG, "doc_terms is NULL");
+  for (int64_t p = 0; p < total; ++p)
+    if (doc_terms[p] < 0 || doc_terms[p] >= vocab)
+      return fail(OPRAG_ERR_INVALID_ARG, "term id %d outside [0, %d)", doc_terms[p], vocab);
+
+  // Term frequencies per chunk, document frequencies, average length.
+  std::vector<int64_t> df(vocab, 0);
+  std::vector<int32_t> tmp;
+  std::vector<int32_t> pair_doc, pair_term, pair_tf;
+  pair_doc.reserve(total);
+  pair_term.reserve(total);
+  pair_tf.reserve(total);
+  for (int64_t dd = 0; dd < n; ++dd) {
+    tmp.assign(doc_terms + doc_indptr[dd], doc_terms + doc_indptr[dd + 1]);
+    std::sort(tmp.begin(), tmp.end());
+    for (size_t i = 0; i < tmp.size();) {
+      size_t j = i;
+      while (j < tmp.size() && tmp[j] == tmp[i]) ++j;
+      pair_doc.push_back(static_cast<int32_t>(dd));
+      pair_term.push_back(tmp[i]);
+      pair_tf.push_back(static_cast<int32_t>(j - i));
+      df[tmp[i]] += 1;
+      i = j;
+    }
+  }
+  const double avgdl = static_cast<double>(total) / static_cast<double>(n);
+  // Postings grouped by term, chunks ascending inside a term.
+  std::vector<int64_t> ptr(static_cast<size_t>(vocab) + 1, 0);
+  for (int t = 0; t < vocab; ++t) ptr[t + 1] = ptr[t] + df[t];
+  const int64_t nnz = ptr[vocab];
+  std::vector<int32_t> pdoc(nnz);
+  std::vector<float> pw(nnz);
+  std::vector<int64_t> fill(ptr.begin(), ptr.end() - 1);
+  const double N = static_cast<double>(n);
+  for (size_t i = 0; i < pair_doc.size(); ++i) {
+    const int32_t t = pair_term[i], dd = pair_doc[i];
+    const double len = static_cast<double>(doc_indptr[dd + 1] - doc_indptr[dd]);
+    const double norm = 1.0 - b + b * (avgdl > 0.0 ? len / avgdl : 0.0);
+    const double dft = static_cast<double>(df[t]);
+    const double idf = std::log(1.0 + (N - dft + 0.5) / (dft + 0.5));
+    const double tf = static_cast<double>(pair_tf[i]);
+    const int64_t at = fill[t]++;
+    pdoc[at] = dd;
+    pw[at] = static_cast<float>(idf * tf * (k1 + 1.0) / (tf + k1 * norm));
+  }
+
+  DeviceGuard g(idx->device);
+  cudaError_t e = idx->drain();
+  if (e != cudaSuccess) return cuda_fail(e, "waiting for pending work");
+  idx->free_sparse();
+  if (cudaMalloc(&idx->post_ptr, ptr.size() * sizeof(int64_t)) != cudaSuccess ||
+      cudaMalloc(&idx->post_doc, std::max<int64_t>(nnz, 1) * sizeof(int32_t)) != cudaSuccess ||
+      cudaMalloc(&idx->post_w, std::max<int64_t>(nnz, 1) * sizeof(float)) != cudaSuccess) {
+    cudaGetLastError();
+    idx->free_sparse();
+    return fail(OPRAG_ERR_OOM, "cannot allocate postings");
+  }
+  e = cudaMemcpy(idx->post_ptr, ptr.data(), ptr.size() * sizeof(int64_t), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && nnz)
+    e = cudaMemcpy(idx->post_doc, pdoc.data(), nnz * sizeof(int32_t), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && nnz)
+    e = cudaMemcpy(idx->post_w, pw.data(), nnz * sizeof(float), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) {
+    idx->free_sparse();
+    return cuda_fail(e, "uploading postings");
+  }
+  idx->vocab = vocab;
+  idx->nnz = nnz;
+  idx->has_sparse = true;
+  return ok();
+}
+
+int oprag_hybrid_search(oprag_index* idx, const void* queries, int32_t q, const int32_t* q_indptr,
+                        const int32_t* q_terms, float alpha, int32_t k, int64_t* out_ids,
+                        float* out_scores, void* stream) {
+  int rc = check_search_args(idx, queries, q, k, out_ids, out_scores);
+  if (rc) return rc;
+  if (!idx->has_sparse) return fail(OPRAG_ERR_NOT_READY, "no sparse side: call oprag_index_set_sparse");
+  if (q == 0) return ok();
+  if (!q_indptr || !q_terms) return fail(OPRAG_ERR_INVALID_ARG, "NULL query terms");
+  if (!std::isfinite(alpha)) return fail(OPRAG_ERR_INVALID_ARG, "alpha is not finite");
+  DeviceGuard g(idx->device);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int64_t ld = (idx->n + 3) / 4 * 4;
+  const int qchunk = static_cast<int>(std::min<int64_t>(q, std::max<int64_t>(1, kLexMaxElems / ld)));
+  if ((rc = idx->ensure(reinterpret_cast<void**>(&idx->lex), &idx->lex_bytes,
+                        sizeof(float) * static_cast<size_t>(qchunk * ld + qchunk), "BM25 block")))
+    return rc;
+  if ((rc = begin_call(idx, st))) return rc;
+  const SparseIndex sp{idx->vocab, idx->nnz, idx->post_ptr, idx->post_doc, idx->post_w};
+  const size_t qrow = static_cast<size_t>(idx->d) * elem_size(idx->dtype);
+  for (int c0 = 0; c0 < q; c0 += qchunk) {
+    const int qc = std::min(qchunk, q - c0);
+    float* lex = idx->lex;
+    float* lexmax = idx->lex + static_cast<size_t>(qc) * ld;
+    if (idx->timing) cudaEventRecord(idx->ev[0], st);
+    idx->timed_lex = idx->timing;
+    cudaError_t e = launch_bm25_matrix(sp, idx->n, q_indptr + c0, q_terms, qc, lex, ld, lexmax, st);
+    if (e != cudaSuccess) return cuda_fail(e, "BM25 kernel");
+    const Fusion fu{lex, ld, lexmax, alpha};
+    if ((rc = run_search(idx, static_cast<const char*>(queries) + c0 * qrow, qc, k, fu,
+                         out_ids + static_cast<size_t>(c0) * k,
+                         out_scores + static_cast<size_t>(c0) * k, st)))
+      return rc;
+  }
+  return end_call(idx, st);
+}
+
+int oprag_index_check(oprag_index* idx) {
+  if (!idx) return fail(OPRAG_ERR_INVALID_ARG, "index is NULL");
+  DeviceGuard g(idx->device);
+  cudaError_t e = idx->drain();
+  if (e != cudaSuccess) return cuda_fail(e, "pending work");
+  int flag = 0;
+  e = cudaMemcpy(&flag, idx->dev_err, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "reading the error word");
+  if (flag != 0) {
+    cudaMemset(idx->dev_err, 0, sizeof(int));
+    return fail(OPRAG_ERR_DEVICE, "a kernel gave up a bounded wait (code %d)", flag);
+  }
+  return ok();
+}
+
+int oprag_index_set_option(oprag_index* idx, int32_t option, int32_t value) {
+  if (!idx) return fail(OPRAG_ERR_INVALID_ARG, "index is NULL");
+  if (option == OPRAG_OPT_PATH) {
+    if (value < 0 || value > 2) return fail(OPRAG_ERR_INVALID_ARG, "path %d", value);
+    if (value == 2 && idx->dtype != OPRAG_BF16)
+      return fail(OPRAG_ERR_INVALID_ARG, "the tensor-core path needs a bf16 index");
+    idx->opt_path = value;
+    return ok();
+  }
+  if (option == OPRAG_OPT_TIMING) {
+    if (value && !idx->ev[0]) {
+      DeviceGuard g(idx->device);
+      for (cudaEvent_t& ev : idx->ev) {
+        cudaError_t e = cudaEventCreate(&ev);
+        if (e != cudaSuccess) return cuda_fail(e, "timing events");
+      }
+    }
+    idx->timing = value != 0;
+    return ok();
+  }
+  if (option == OPRAG_OPT_BLOCK_N) {
+    if (value != 0 && value != 64 && value != 256)
+      return fail(OPRAG_ERR_INVALID_ARG, "block_n %d", value);
+    idx->opt_block_n = value;
+    return ok();
+  }
+  return fail(OPRAG_ERR_INVALID_ARG, "unknown option %d", option);
+}
+
+int oprag_index_last_path(const oprag_index* idx) { return idx ? idx->last_path : 0; }
+
+int oprag_index_last_timing(oprag_index* idx, float* lexical_ms, float* search_ms,
+                            float* merge_ms) {
+  if (!idx) return fail(OPRAG_ERR_INVALID_ARG, "index is NULL");
+  if (!idx->timed) return fail(OPRAG_ERR_NOT_READY, "no timed search was issued");
+  DeviceGuard g(idx->device);
+  cudaError_t e = cudaEventSynchronize(idx->ev[3]);
+  if (e != cudaSuccess) return cuda_fail(e, "timing");
+  float a = 0.f, b = 0.f, c = 0.f;
+  if (idx->timed_lex) e = cudaEventElapsedTime(&a, idx->ev[0], idx->ev[1]);
+  if (e == cudaSuccess) e = cudaEventElapsedTime(&b, idx->ev[1], idx->ev[2]);
+  if (e == cudaSuccess) e = cudaEventElapsedTime(&c, idx->ev[2], idx->ev[3]);
+  if (e != cudaSuccess) return cuda_fail(e, "timing");
+  if (lexical_ms) *lexical_ms = a;
+  if (search_ms) *search_ms = b;
+  if (merge_ms) *merge_ms = c;
+  return ok();
+}
+
+}  // extern "C"

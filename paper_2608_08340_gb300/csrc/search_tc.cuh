@@ -1,0 +1,480 @@
+// Tensor-core search for bf16 indices on sm_103a: the query x chunk score
+// contraction of Sec. 4.4 ("dense scores ... vectorized matrix operations
+// over the embedding matrix") as a tcgen05 GEMM, with the partial top-k
+// selection (Sec. 4.4, Sec. 7) fused into the epilogue so that the q x n
+// score matrix never reaches HBM.
+//
+// Work decomposition.  Queries are cut into tiles of 128 (the MMA M side, one
+// query per TMEM lane) and the corpus into tiles of BN rows (the MMA N side).
+// A unit is (corpus tile t, query tile j), numbered u = t * QT + j, and CTA c
+// of a persistent grid of C CTAs takes units c, c + C, c + 2C, ...  All CTAs
+// therefore sweep the corpus together, each corpus tile being read by the QT
+// CTAs that need it at about the same time (one HBM read, QT - 1 L2 hits).
+// CTA c meets the query tiles j == c (mod g), g = gcd(C, QT); it keeps one
+// running top-K list per query for each of them ("slots") and leaves it as
+// partial list p = c / g of tile j for the merge kernel.
+//
+// Roles (192 threads):
+//   warp 0, lane 0: TMA producer.  Per K block of 64 bf16 (one 128-byte
+//                   swizzle row) it loads the 128 x 64 query tile and the
+//                   BN x 64 corpus tile into a pipeline stage.
+//   warp 1        : allocates 2 x BN TMEM columns (two fp32 accumulators);
+//                   lane 0 issues tcgen05.mma (M = 128, N = BN, K = 16).
+//   warps 2..5    : epilogue.  Each thread owns one query (one TMEM lane),
+//                   reads its BN scores with tcgen05.ld and filters them
+//                   against its running k-th best score.
+// The two accumulators let the epilogue of one unit overlap the MMAs of the
+// next.  Every mbarrier wait is bounded (see common.cuh).
+#pragma once
+#include <cuda.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace oprag {
+namespace tc {
+
+constexpr int kBlockM = 128;
+constexpr int kBlockK = 64;                 // bf16 per 128-byte row
+constexpr int kUmmaK = 16;
+constexpr int kThreads = 192;
+constexpr uint32_t kAStageBytes = kBlockM * kBlockK * 2;
+constexpr int kSmemBudget = 200 * 1024;
+
+struct TcParams {
+  int64_t n;
+  int d;
+  int q;
+  int k;
+  int qt;
+  int64_t units;
+  int g;
+  int P;
+  int slots;
+  int kblocks;
+  Fusion fu;
+  uint64_t* lists;      // [(j * P + p) * 128 + row] * stride
+  int* meta_count;      // buffered lists: kept keys per (list, row)
+  uint64_t* meta_worst; // buffered lists: K-th key per (list, row)
+  int* dev_err;
+};
+
+template <int BN>
+constexpr int stages_for() {
+  return kSmemBudget / (kAStageBytes + BN * 128) > 8 ? 8 : kSmemBudget / (kAStageBytes + BN * 128);
+}
+
+template <int BN>
+constexpr size_t smem_for() {
+  return static_cast<size_t>(stages_for<BN>()) * (kAStageBytes + BN * 128) + 1024 + 256;
+}
+
+// ----------------------------------------------------------------- PTX
+
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x,
+                                            int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_addr(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_addr(bar)), "r"(x), "r"(y)
+      : "memory");
+}
+
+__device__ __forceinline__ void prefetch_map(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_addr(slot)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand in the 128-byte swizzle
+// layout written by TMA (8-row groups 1024 bytes apart).
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  uint64_t desc = 0;
+  desc |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);   // start address
+  desc |= static_cast<uint64_t>(1) << 16;                    // leading byte offset (unused)
+  desc |= static_cast<uint64_t>(1024 >> 4) << 32;            // stride byte offset
+  desc |= static_cast<uint64_t>(1) << 46;                    // descriptor version
+  desc |= static_cast<uint64_t>(2) << 61;                    // 128-byte swizzle
+  return desc;
+}
+
+// Instruction descriptor, kind::f16: bf16 A and B (both K-major), fp32 D.
+__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(n >> 3) << 17) |
+         (static_cast<uint32_t>(m >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_addr(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+        "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+        "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Waits without looking at the abort word (used to drain in-flight copies and
+// MMAs before the CTA exits); still bounded.
+__device__ __forceinline__ bool mbar_drain(uint64_t* bar, uint32_t parity, int* dev_err) {
+  const long long t0 = clock64();
+  while (!mbar_test(bar, parity)) {
+    if (clock64() - t0 > kWaitLimitCycles) {
+      atomicExch(dev_err, static_cast<int>(kDevErrWaitTimeout));
+      return false;
+    }
+  }
+  return true;
+}
+
+// ----------------------------------------------------------------- lists
+
+template <int K, bool kBuf = (K > 32)>
+struct EpiList;
+
+template <int K>
+struct EpiList<K, false> {
+  static constexpr int kStride = K;
+  RegTopK<K> t;
+  __device__ __forceinline__ void init_mem(const TcParams& p, int64_t sr) {
+#pragma unroll
+    for (int i = 0; i < K; i += 2)
+      *reinterpret_cast<ulonglong2*>(p.lists + sr * K + i) = make_ulonglong2(0ull, 0ull);
+  }
+  __device__ __forceinline__ void load(const TcParams& p, int64_t sr) { t.load(p.lists + sr * K); }
+  __device__ __forceinline__ void save(const TcParams& p, int64_t sr) { t.store(p.lists + sr * K); }
+  __device__ __forceinline__ void clear() { t.init(); }
+  __device__ __forceinline__ float floor() const { return t.floor; }
+  __device__ __forceinline__ void push(float s, uint32_t id) { t.push(s, id); }
+  __device__ __forceinline__ void sync(bool, bool) {}
+  __device__ __forceinline__ void finalize(const TcParams&, int64_t, bool) {}
+};
+
+template <int K>
+struct EpiList<K, true> {
+  static constexpr int kStride = 2 * K;
+  BufTopK<K> t;
+  __device__ __forceinline__ void init_mem(const TcParams& p, int64_t sr) {
+    p.meta_count[sr] = 0;
+    p.meta_worst[sr] = kEmptyKey;
+  }
+  __device__ __forceinline__ void load(const TcParams& p, int64_t sr) {
+    t.buf = p.lists + sr * kStride;
+    t.count = p.meta_count[sr];
+    t.worst = p.meta_worst[sr];
+    t.floor = key_floor(t.worst);
+  }
+  __device__ __forceinline__ void save(const TcParams& p, int64_t sr) {
+    p.meta_count[sr] = t.count;
+    p.meta_worst[sr] = t.worst;
+  }
+  __device__ __forceinline__ void clear() {
+    t.buf = nullptr;
+    t.count = 0;
+    t.worst = kEmptyKey;
+    t.floor = -INFINITY;
+  }
+  __device__ __forceinline__ float floor() const { return t.floor; }
+  __device__ __forceinline__ void push(float s, uint32_t id) { t.push(s, id); }
+  __device__ __forceinline__ void sync(bool final, bool active) { t.sync(final, active); }
+  // Warp-collective: sorts the lane's buffer, best K first.
+  __device__ __forceinline__ void finalize(const TcParams& p, int64_t sr, bool valid) {
+    if (valid) load(p, sr); else clear();
+    t.sync(true, valid);
+  }
+};
+
+// ----------------------------------------------------------------- kernel
+
+template <int BN, int K, bool kHybrid>
+__global__ void __launch_bounds__(kThreads, 1)
+tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_e,
+                 const TcParams p) {
+  constexpr int S = stages_for<BN>();
+  constexpr uint32_t kBStageBytes = BN * 128;
+  constexpr uint32_t kTmemCols = 2 * BN;
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  unsigned char* base = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  unsigned char* sA = base;
+  unsigned char* sB = sA + S * kAStageBytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sB + S * kBStageBytes);
+  uint64_t* empty = full + S;
+  uint64_t* tfull = empty + S;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* mma_done = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int cta = blockIdx.x, C = gridDim.x;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);
+      mbar_init(&tempty[b], 4);
+    }
+    mbar_init(mma_done, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    prefetch_map(&map_q);
+    prefetch_map(&map_e);
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------ TMA producer
+      int s = 0;
+      uint32_t ph = 0;
+      uint32_t issued = 0, parity = 0;    // per stage: ever issued, parity of last issue
+      bool ok = true;
+      for (int64_t u = cta; ok && u < p.units; u += C) {
+        const int j = static_cast<int>(u % p.qt);
+        const int t = static_cast<int>(u / p.qt);
+        for (int kb = 0; kb < p.kblocks; ++kb) {
+          if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, p.dev_err)) { ok = false; break; }
+          mbar_arrive_expect_tx(&full[s], kAStageBytes + kBStageBytes);
+          tma_load_2d(sA + s * kAStageBytes, &map_q, &full[s], kb * kBlockK, j * kBlockM);
+          tma_load_2d(sB + s * kBStageBytes, &map_e, &full[s], kb * kBlockK, t * BN);
+          issued |= 1u << s;
+          parity = (parity & ~(1u << s)) | (ph << s);
+          if (++s == S) { s = 0; ph ^= 1u; }
+        }
+      }
+      for (int i = 0; i < S; ++i)
+        if (issued & (1u << i)) mbar_drain(&full[i], (parity >> i) & 1u, p.dev_err);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------ MMA issuer
+      constexpr uint32_t idesc = idesc_bf16(kBlockM, BN);
+      int s = 0;
+      uint32_t ph = 0;
+      int acc = 0;
+      uint32_t acc_ph = 0;
+      bool ok = true;
+      for (int64_t u = cta; ok && u < p.units; u += C) {
+        if (!mbar_wait(&tempty[acc], acc_ph ^ 1u, abort_flag, p.dev_err)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
+        for (int kb = 0; kb < p.kblocks; ++kb) {
+          if (!mbar_wait(&full[s], ph, abort_flag, p.dev_err)) { ok = false; break; }
+          tc_fence_after();
+          const uint64_t a = sw128_desc(smem_addr(sA + s * kAStageBytes));
+          const uint64_t b = sw128_desc(smem_addr(sB + s * kBStageBytes));
+#pragma unroll
+          for (int kk = 0; kk < kBlockK / kUmmaK; ++kk)
+            mma_bf16(d_tmem, a + 2 * kk, b + 2 * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
+          mma_commit(&empty[s]);
+          if (++s == S) { s = 0; ph ^= 1u; }
+        }
+        if (!ok) break;
+        mma_commit(&tfull[acc]);
+        if (++acc == 2) { acc = 0; acc_ph ^= 1u; }
+      }
+      mma_commit(mma_done);
+      mbar_drain(mma_done, 0, p.dev_err);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------ epilogue
+    const int eg = warp & 3;                 // TMEM lane group of this warp
+    const int row = eg * 32 + lane;          // query row within a tile
+    const int c_mod = cta % p.g, my_p = cta / p.g;
+    EpiList<K> list;
+    list.clear();
+
+    for (int s = 0; s < p.slots; ++s) {
+      const int j = c_mod + s * p.g;
+      if (j * kBlockM + row < p.q) list.init_mem(p, (static_cast<int64_t>(j) * p.P + my_p) * kBlockM + row);
+    }
+
+    int cur_slot = -1;
+    int64_t cur_sr = 0;
+    bool cur_valid = false;
+    int acc = 0;
+    uint32_t acc_ph = 0;
+    for (int64_t u = cta; u < p.units; u += C) {
+      const int j = static_cast<int>(u % p.qt);
+      const int64_t t = u / p.qt;
+      const int slot = (j - c_mod) / p.g;
+      const bool valid = j * kBlockM + row < p.q;
+      const bool warp_live = j * kBlockM + eg * 32 < p.q;
+      if (slot != cur_slot) {
+        if (cur_slot >= 0 && cur_valid) list.save(p, cur_sr);
+        cur_slot = slot;
+        cur_sr = (static_cast<int64_t>(j) * p.P + my_p) * kBlockM + row;
+        cur_valid = valid;
+        if (valid) list.load(p, cur_sr); else list.clear();
+      }
+      if (!mbar_wait(&tfull[acc], acc_ph, abort_flag, p.dev_err)) break;
+      tc_fence_after();
+      if (warp_live) {
+        float inv_max = 0.f;
+        const float* brow = nullptr;
+        if (kHybrid && valid) {
+          const float m = p.fu.bm25_max[j * kBlockM + row];
+          inv_max = m > 0.f ? 1.f / m : 0.f;
+          brow = p.fu.bm25 + static_cast<int64_t>(j * kBlockM + row) * p.fu.ld;
+        }
+        const uint32_t taddr = tmem_base + (static_cast<uint32_t>(eg * 32) << 16) +
+                               static_cast<uint32_t>(acc * BN);
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          float v[32];
+          __syncwarp();
+          tmem_ld32(taddr + c * 32, v);
+          const int64_t id0 = t * BN + c * 32;
+          if (kHybrid && valid) {
+            const float a = p.fu.alpha, b1 = 1.f - p.fu.alpha;
+            if (id0 + 32 <= p.n) {
+#pragma unroll
+              for (int i = 0; i < 32; i += 4) {
+                const float4 w = *reinterpret_cast<const float4*>(brow + id0 + i);
+                v[i] = fmaf(a, v[i], b1 * (w.x * inv_max));
+                v[i + 1] = fmaf(a, v[i + 1], b1 * (w.y * inv_max));
+                v[i + 2] = fmaf(a, v[i + 2], b1 * (w.z * inv_max));
+                v[i + 3] = fmaf(a, v[i + 3], b1 * (w.w * inv_max));
+              }
+            } else {
+#pragma unroll
+              for (int i = 0; i < 32; ++i)
+                if (id0 + i < p.n) v[i] = fmaf(a, v[i], b1 * (brow[id0 + i] * inv_max));
+            }
+          }
+          if (id0 + 32 > p.n) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if (id0 + i >= p.n) v[i] = -INFINITY;
+          }
+          list.sync(false, valid);
+          float m = v[0];
+#pragma unroll
+          for (int i = 1; i < 32; ++i) m = fmaxf(m, v[i]);
+          if (valid && m >= list.floor()) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i)
+              if (v[i] >= list.floor()) list.push(v[i], static_cast<uint32_t>(id0 + i));
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[acc]);
+      if (++acc == 2) { acc = 0; acc_ph ^= 1u; }
+    }
+    if (cur_slot >= 0 && cur_valid) list.save(p, cur_sr);
+    if (K > 32) {
+      for (int s = 0; s < p.slots; ++s) {
+        const int j = c_mod + s * p.g;
+        const bool valid = j * kBlockM + row < p.q;
+        list.finalize(p, (static_cast<int64_t>(j) * p.P + my_p) * kBlockM + row, valid);
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem_base, kTmemCols);
+}
+
+// ----------------------------------------------------------------- launch
+
+template <int BN, int K, bool H>
+cudaError_t launch_variant(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
+                           int grid, cudaStream_t st) {
+  constexpr size_t smem = smem_for<BN>();
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(tc_search_kernel<BN, K, H>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  tc_search_kernel<BN, K, H><<<grid, kThreads, smem, st>>>(mq, me, prm);
+  return cudaGetLastError();
+}
+
+template <int BN, int K>
+cudaError_t launch_k(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm, int grid,
+                     bool hybrid, cudaStream_t st) {
+  return hybrid ? launch_variant<BN, K, true>(mq, me, prm, grid, st)
+                : launch_variant<BN, K, false>(mq, me, prm, grid, st);
+}
+
+template <int BN>
+cudaError_t launch_bn(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm, int grid,
+                      bool hybrid, cudaStream_t st) {
+  switch (list_len_for(prm.k)) {
+    case 8: return launch_k<BN, 8>(mq, me, prm, grid, hybrid, st);
+    case 32: return launch_k<BN, 32>(mq, me, prm, grid, hybrid, st);
+    case 128: return launch_k<BN, 128>(mq, me, prm, grid, hybrid, st);
+    default: return launch_k<BN, 256>(mq, me, prm, grid, hybrid, st);
+  }
+}
+
+// Instantiations live in their own translation units (parallel builds).
+cudaError_t launch_bn64(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm, int grid,
+                        bool hybrid, cudaStream_t st);
+cudaError_t launch_bn256_dense(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
+                               int grid, cudaStream_t st);
+cudaError_t launch_bn256_fused(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
+                               int grid, cudaStream_t st);
+
+}  // namespace tc
+}  // namespace oprag

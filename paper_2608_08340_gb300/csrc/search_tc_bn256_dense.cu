@@ -1,0 +1,18 @@
+// Tensor-core search kernels with 256-row corpus tiles, dense scores.
+#include "search_tc.cuh"
+
+namespace oprag {
+namespace tc {
+
+cudaError_t launch_bn256_dense(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
+                               int grid, cudaStream_t st) {
+  switch (list_len_for(prm.k)) {
+    case 8: return launch_variant<256, 8, false>(mq, me, prm, grid, st);
+    case 32: return launch_variant<256, 32, false>(mq, me, prm, grid, st);
+    case 128: return launch_variant<256, 128, false>(mq, me, prm, grid, st);
+    default: return launch_variant<256, 256, false>(mq, me, prm, grid, st);
+  }
+}
+
+}  // namespace tc
+}  // namespace oprag

@@ -1,0 +1,198 @@
+"""GPU parity of the dense search (both kernel families) against the fp64
+oracle: hand-worked fixture, the paper-shaped workloads, ragged shapes that
+span several tiles, ties and degenerate inputs.  Scores must be within 1e-4 of
+the oracle; ids must match except inside near-tie blocks (oracle/check.py)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from oracle import check
+from paper_2608_08340_gb300 import workloads
+from paper_2608_08340_gb300.index import Index
+
+from _golden import load
+from _gpu import TOL, check_dense, dev_tensor
+
+pytestmark = pytest.mark.gpu
+
+
+def _index(data, dtype=None):
+    return Index(dev_tensor(data), dtype)
+
+
+@pytest.mark.parametrize("dtype,path", [("f32", None), ("bf16", "simt"), ("bf16", "tc")])
+def test_golden_hand_worked(dtype, path):
+    g = load("dense_8chunk.json")
+    E = np.asarray(g["E"], np.float32)
+    Q = np.asarray(g["Q"], np.float32)
+    if dtype == "bf16":
+        E, Q = oracle.round_bf16(E), oracle.round_bf16(Q)
+    idx = _index(E)
+    if path:
+        idx.force_path(path)
+    ids, sc = idx.search(dev_tensor(Q), g["k"])
+    assert ids.cpu().tolist() == g["ids"]
+    assert sc.cpu().tolist() == [[float(v) for v in r] for r in g["scores"]]
+    if path:
+        assert idx.last_path == path
+
+
+def test_config0_tiny_fp32():
+    w = workloads.config(0)
+    idx = _index(w.E_data)
+    ids, sc = idx.search(dev_tensor(w.Q_data), w.k)
+    assert idx.last_path == "simt"
+    check_dense(ids, sc, w.E_data, w.Q_data, w.k, "cfg0")
+
+
+@pytest.fixture(scope="module")
+def cfg1():
+    w = workloads.config(1, batch=256)
+    return w, _index(w.E_data)
+
+
+@pytest.mark.parametrize("q", [1, 32, 256])
+@pytest.mark.parametrize("path", [None, "simt", "tc"])
+def test_config1_paper_shaped(cfg1, q, path):
+    w, idx = cfg1
+    idx.force_path(path)
+    try:
+        ids, sc = idx.search(dev_tensor(w.Q_data[:q]), w.k)
+        torch.cuda.synchronize()
+    finally:
+        idx.force_path(None)
+    check_dense(ids, sc, w.E_data, w.Q_data[:q], w.k, f"cfg1 q={q} path={path}")
+    idx.check()
+
+
+@pytest.mark.parametrize("n,d,q,k", [
+    (1000, 64, 3, 5),          # n not a multiple of any tile
+    (4097, 136, 17, 10),       # d not a multiple of the 64-wide K block
+    (300, 384, 129, 100),      # k close to n, q just past one query tile
+    (5000, 128, 257, 1),       # k = 1, three query tiles
+    (2000, 256, 2, 256),       # k = K_MAX
+    (700, 64, 255, 33),        # list length 128 for k = 33
+])
+@pytest.mark.parametrize("path", ["simt", "tc"])
+def test_ragged_shapes(n, d, q, k, path):
+    rng = np.random.default_rng(n + d + q + k)
+    E = workloads.to_bf16_bits(workloads._normalise(rng.standard_normal((n, d)).astype(np.float32)))
+    Q = workloads.to_bf16_bits(workloads._normalise(rng.standard_normal((q, d)).astype(np.float32)))
+    idx = _index(E)
+    idx.force_path(path)
+    ids, sc = idx.search(dev_tensor(Q), k)
+    assert idx.last_path == path
+    check_dense(ids, sc, E, Q, k, f"ragged n={n} d={d} q={q} k={k} {path}")
+
+
+@pytest.mark.parametrize("bn", [64, 256])
+def test_tc_tile_widths_agree(bn):
+    w = workloads.config(1, n=9000, batch=300)
+    idx = _index(w.E_data)
+    idx.force_path("tc")
+    idx.force_block_n(bn)
+    ids, sc = idx.search(dev_tensor(w.Q_data), 10)
+    check_dense(ids, sc, w.E_data, w.Q_data, 10, f"bn={bn}")
+
+
+@pytest.mark.parametrize("path", ["simt", "tc"])
+def test_duplicate_rows_tie_to_lower_id(path):
+    rng = np.random.default_rng(5)
+    base = rng.standard_normal((64, 128)).astype(np.float32)
+    E = np.concatenate([base, base, base])          # every row three times
+    Eb = oracle.round_bf16(E)
+    Qb = Eb[[3, 70, 150]]
+    idx = _index(Eb)
+    idx.force_path(path)
+    ids, sc = idx.search(dev_tensor(Qb), 3)
+    ids = ids.cpu().numpy()
+    sc = sc.cpu().numpy()
+    for i, r in enumerate([3, 70, 150]):
+        assert ids[i].tolist() == [r % 64, r % 64 + 64, r % 64 + 128]
+        assert sc[i, 0] == sc[i, 1] == sc[i, 2]
+
+
+@pytest.mark.parametrize("path", ["simt", "tc"])
+def test_all_scores_equal_returns_lowest_ids(path):
+    E = oracle.round_bf16(np.ones((500, 64), np.float32))
+    Q = np.zeros((5, 64), np.uint16)                  # zero queries: every score is 0
+    idx = _index(E)
+    idx.force_path(path)
+    ids, sc = idx.search(dev_tensor(Q), 7)
+    assert ids.cpu().tolist() == [list(range(7))] * 5
+    assert (sc.cpu().numpy() == 0).all()
+
+
+def test_k_equal_n_is_full_sort():
+    w = workloads.config(0, n=200, batch=4)
+    idx = _index(w.E_data)
+    ids, sc = idx.search(dev_tensor(w.Q_data), 200)
+    check_dense(ids, sc, w.E_data, w.Q_data, 200, "k=n")
+
+
+def test_argument_errors():
+    w = workloads.config(0, n=100, batch=2)
+    idx = _index(w.E_data)
+    Q = dev_tensor(w.Q_data)
+    for k in (0, 101, 257):
+        with pytest.raises(Exception):
+            idx.search(Q, k)
+    ids, sc = idx.search(Q[:0], 5)                    # q = 0 is a no-op
+    assert ids.shape == (0, 5)
+    with pytest.raises(Exception):
+        idx.search(Q.to(torch.bfloat16), 5)           # dtype mismatch
+
+
+def test_search_host_matches_device_search():
+    w = workloads.config(1, n=8192, batch=40)
+    idx = _index(w.E_data)
+    Qd = dev_tensor(w.Q_data)
+    ids_d, sc_d = idx.search(Qd, 5)
+    ids_h, sc_h = idx.search_host(Qd.cpu().pin_memory(), 5)
+    assert torch.equal(ids_d.cpu(), ids_h)
+    assert torch.equal(sc_d.cpu(), sc_h)
+
+
+def test_fp32_input_into_bf16_index_rounds_to_nearest_even():
+    w = workloads.config(0, n=512, batch=4)        # fp32 data
+    idx = Index(dev_tensor(w.E_data), torch.bfloat16)
+    got = idx.rows().view(torch.int16).numpy().view(np.uint16)
+    np.testing.assert_array_equal(got, oracle.round_bf16(w.E_data))
+    idx2 = Index(torch.from_numpy(w.E_data), torch.bfloat16)   # from host memory
+    got2 = idx2.rows().view(torch.int16).numpy().view(np.uint16)
+    np.testing.assert_array_equal(got2, got)
+
+
+def test_config2_clustered_near_ties_sampled():
+    w = workloads.config(2)
+    idx = _index(w.E_data)
+    ids, sc = idx.search(dev_tensor(w.Q_data), w.k)
+    assert idx.last_path == "tc"
+    rows = np.random.default_rng(0).choice(w.q, 48, replace=False)
+    rows.sort()
+    check_dense(ids, sc, w.E_data, w.Q_data, w.k, "cfg2", rows=rows)
+
+
+@pytest.mark.slow
+def test_config4_scale_with_upserts_sampled():
+    """1M x 768 bf16, 4 batches of 2048 queries, 4096-row upserts before
+    batches 2-4; sampled queries of every batch checked against the oracle
+    run on the post-upsert index."""
+    w = workloads.config(4, batch=8192)
+    E = w.E_data.copy()
+    idx = _index(E)
+    rng = np.random.default_rng(1)
+    for b in range(4):
+        if b > 0:
+            up_ids, up_rows = workloads.upsert_batch(w.n, w.d, 4096, b, "bf16")
+            idx.upsert(up_ids, dev_tensor(up_rows))
+            oracle.upsert(E, up_ids, up_rows)
+        Qb = w.Q_data[b * 2048:(b + 1) * 2048]
+        ids, sc = idx.search(dev_tensor(Qb), w.k)
+        rows = np.sort(rng.choice(2048, 6, replace=False))
+        check_dense(ids, sc, E, Qb, w.k, f"cfg4 batch {b}", rows=rows)
+    # the index equals the oracle's post-upsert array
+    got = idx.rows().view(torch.int16).numpy().view(np.uint16)
+    np.testing.assert_array_equal(got, E)
+    idx.check()
