@@ -161,6 +161,81 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+class NvmlSampler:
+    """Reads SM clock and clock-event reasons through NVML every 2 ms on a
+    background thread (read-only queries; nothing is set)."""
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, torch_device: int):
+        import ctypes
+        import threading
+        self.samples = []
+        self.max_mhz = None
+        self.error = None
+        self._stop = threading.Event()
+        self._thread = None
+        try:
+            import torch
+            lib = ctypes.CDLL("libnvidia-ml.so.1")
+            if lib.nvmlInit_v2() != 0:
+                raise RuntimeError("nvmlInit failed")
+            self.lib = lib
+            self.h = ctypes.c_void_p()
+            props = torch.cuda.get_device_properties(torch_device)
+            ok = False
+            for attr in ("pci_domain_id", "pci_bus_id", "pci_device_id"):
+                if not hasattr(props, attr):
+                    break
+            else:
+                bus = f"{props.pci_domain_id:08x}:{props.pci_bus_id:02x}:{props.pci_device_id:02x}.0"
+                ok = lib.nvmlDeviceGetHandleByPciBusId_v2(bus.encode(), ctypes.byref(self.h)) == 0
+            if not ok and lib.nvmlDeviceGetHandleByIndex_v2(torch_device, ctypes.byref(self.h)) != 0:
+                raise RuntimeError("no NVML handle")
+            mx = ctypes.c_uint()
+            if lib.nvmlDeviceGetMaxClockInfo(self.h, 1, ctypes.byref(mx)) == 0:
+                self.max_mhz = float(mx.value)
+            self.get_reasons = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+                lib.nvmlDeviceGetCurrentClocksThrottleReasons
+        except Exception as e:  # noqa: BLE001
+            self.error = str(e)
+
+    def _run(self):
+        import ctypes
+        clk = ctypes.c_uint()
+        rs = ctypes.c_ulonglong()
+        while not self._stop.is_set():
+            if self.lib.nvmlDeviceGetClockInfo(self.h, 1, ctypes.byref(clk)) == 0:
+                r = rs.value if self.get_reasons(self.h, ctypes.byref(rs)) == 0 else 0
+                self.samples.append((float(clk.value), int(r)))
+            self._stop.wait(0.002)
+
+    def __enter__(self):
+        import threading
+        if self.error is None:
+            self._thread = threading.Thread(target=self._run, daemon=True)
+            self._thread.start()
+        return self
+
+    def __exit__(self, *exc):
+        self._stop.set()
+        if self._thread is not None:
+            self._thread.join(timeout=2)
+
+    def summary(self):
+        if self.error is not None or not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": self.max_mhz, "reasons": [],
+                    "samples": 0, "source": f"nvml unavailable: {self.error}"}
+        reasons = set()
+        for _, r in self.samples:
+            for bit, name in self.REASONS.items():
+                if r & bit:
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(c for c, _ in self.samples),
+                "sm_max_mhz": self.max_mhz, "reasons": sorted(reasons),
+                "samples": len(self.samples), "source": "nvml, 2 ms, timed region"}
+
+
 def make_inputs(cfg: int, batch: int):
     if cfg == 4:
         w = workloads.config(4, batch=batch)
@@ -237,7 +312,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
         torch.distributed.barrier()
     torch.cuda.synchronize()
     step_ms, search_ms, lex_ms, merge_ms = [], [], [], []
-    with ClockSampler(local_rank) as clocks:
+    with ClockSampler(local_rank) as smi, NvmlSampler(local_rank) as clocks:
         for i in range(args.steps):
             flush.zero_()
             a = torch.cuda.Event(enable_timing=True)
@@ -336,7 +411,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "api": "oprag_search_host" if cfg != 3 else "oprag_hybrid_search + torch copies"},
         "gpu_launches": launches_per_step * args.steps,
-        "clocks": clocks.summary(),
+        "clocks": dict(clocks.summary(), smi=smi.summary()),
         "path": idx.last_path,
     }
     idx.close()

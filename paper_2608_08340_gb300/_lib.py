@@ -63,7 +63,8 @@ class OpragError(RuntimeError):
 
 
 def library_path() -> str:
-    return _build.LIB_PATH
+    """The in-tree library, or the file named by $OPRAG_LIBRARY."""
+    return os.environ.get("OPRAG_LIBRARY") or _build.LIB_PATH
 
 
 def load(path: str | None = None) -> ctypes.CDLL:

@@ -10,9 +10,11 @@ namespace oprag {
 
 enum Dtype : int { kF32 = 0, kBF16 = 1 };
 
-// Kept-list length used for a requested k: 8 or 32 (register lists), 128 or
-// 256 (buffered lists).
-inline int list_len_for(int k) { return k <= 8 ? 8 : k <= 32 ? 32 : k <= 128 ? 128 : 256; }
+// Kept-list length used for a requested k: 8, 16 or 32 (register lists), 128
+// or 256 (buffered lists).
+inline int list_len_for(int k) {
+  return k <= 8 ? 8 : k <= 16 ? 16 : k <= 32 ? 32 : k <= 128 ? 128 : 256;
+}
 
 // Partial top-K lists written by a search kernel and read by the merge.  The
 // list of query row `row` of query tile `tile` produced by producer `p` starts

@@ -3,6 +3,12 @@
 // This is the "local candidates, then global top-k reduction" step of
 // Op_retrieve (Sec. 3.2; Sec. 4.1 Retrieval), done inside one GPU: the
 // producers are corpus slices instead of index shards.
+//
+// One CTA per query.  The P * k candidate keys of a query (the first k of each
+// producer's sorted list) are split evenly over the warps; a warp fetches four
+// 32-key groups at once (independent loads, so L2 latency is paid once per
+// group of four, not once per list) and filters them against its running
+// k-th best.  Warp 0 then merges the warps' results.
 #include "common.cuh"
 #include "internal.h"
 
@@ -11,9 +17,19 @@ namespace oprag {
 namespace {
 
 constexpr int kMergeWarps = 8;
+constexpr int kUnroll = 4;
 
-// One CTA per query.  Warp w merges producers w, w+8, ... into its own buffer;
-// warp 0 then merges the eight warp results and writes the answer.
+template <int KP>
+__device__ __forceinline__ void offer32(WarpMerger<KP>& m, uint64_t key) {
+  const int lane = threadIdx.x & 31;
+  const bool pass = key > m.worst;
+  const uint32_t bits = __ballot_sync(0xffffffffu, pass);
+  if (bits == 0) return;
+  if (m.count > WarpMerger<KP>::kCap - 32) m.compact();
+  if (pass) m.sbuf[m.count + __popc(bits & ((1u << lane) - 1u))] = key;
+  m.count += __popc(bits);
+}
+
 template <int KP>
 __global__ void __launch_bounds__(kMergeWarps * 32)
 merge_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
@@ -24,14 +40,27 @@ merge_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
   if (qi >= q) return;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int tile = qi / ls.TH, row = qi % ls.TH;
+  const uint64_t* base = ls.keys + (static_cast<int64_t>(tile) * ls.P * ls.TH + row) * ls.stride;
+  const int64_t list_step = static_cast<int64_t>(ls.TH) * ls.stride;
+  const int total = ls.P * k;
+  const int lo = static_cast<int>(static_cast<int64_t>(total) * warp / kMergeWarps);
+  const int hi = static_cast<int>(static_cast<int64_t>(total) * (warp + 1) / kMergeWarps);
 
   WarpMerger<KP> m;
   m.init(smem_keys + warp * kCap, k);
-  for (int p = warp; p < ls.P; p += kMergeWarps) {
-    const uint64_t* list =
-        ls.keys + (static_cast<int64_t>(tile) * ls.P + p) * ls.TH * ls.stride +
-        static_cast<int64_t>(row) * ls.stride;
-    m.offer_list(list, k);
+  for (int g = lo; g < hi; g += 32 * kUnroll) {
+    uint64_t key[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int i = g + u * 32 + lane;
+      key[u] = kEmptyKey;
+      if (i < hi) {
+        const int p = i / k;
+        key[u] = base[p * list_step + (i - p * k)];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) offer32(m, key[u]);
   }
   m.finish();
   __syncthreads();
@@ -39,7 +68,21 @@ merge_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
 
   WarpMerger<KP> f;
   f.init(smem_keys + kMergeWarps * kCap, k);
-  for (int w = 0; w < kMergeWarps; ++w) f.offer_list(smem_keys + w * kCap, k);
+  const int all = kMergeWarps * k;
+  for (int g = 0; g < all; g += 32 * kUnroll) {
+    uint64_t key[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const int i = g + u * 32 + lane;
+      key[u] = kEmptyKey;
+      if (i < all) {
+        const int w = i / k;
+        key[u] = smem_keys[w * kCap + (i - w * k)];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) offer32(f, key[u]);
+  }
   f.finish();
   for (int i = lane; i < k; i += 32) {
     const uint64_t key = f.sbuf[i];

@@ -9,7 +9,7 @@
 #include <unordered_set>
 #include <vector>
 
-#include "../../include/oprag.h"
+#include "oprag.h"
 #include "internal.h"
 
 using namespace oprag;

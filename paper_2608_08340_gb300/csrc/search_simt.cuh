@@ -255,6 +255,7 @@ cudaError_t launch_qc(const void* E, const void* Q, const SearchShape& s, const 
                       void* scratch, int grid, ListSet* lists, cudaStream_t st) {
   switch (list_len_for(s.k)) {
     case 8: return launch_t<T, QC, 8>(E, Q, s, fu, scratch, grid, lists, st);
+    case 16: return launch_t<T, QC, 16>(E, Q, s, fu, scratch, grid, lists, st);
     case 32: return launch_t<T, QC, 32>(E, Q, s, fu, scratch, grid, lists, st);
     case 128: return launch_t<T, QC, 128>(E, Q, s, fu, scratch, grid, lists, st);
     default: return launch_t<T, QC, 256>(E, Q, s, fu, scratch, grid, lists, st);

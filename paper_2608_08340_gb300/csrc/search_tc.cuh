@@ -404,10 +404,25 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
           float m = v[0];
 #pragma unroll
           for (int i = 1; i < 32; ++i) m = fmaxf(m, v[i]);
-          if (valid && m >= list.floor()) {
+          const float fl = list.floor();
+          if (__any_sync(0xffffffffu, valid && m >= fl)) {
+            // Lanes insert their candidates together, one column per round,
+            // so the warp runs max-per-lane rounds instead of the sum.
+            uint32_t mask = 0;
+            if (valid) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i)
-              if (v[i] >= list.floor()) list.push(v[i], static_cast<uint32_t>(id0 + i));
+              for (int i = 0; i < 32; ++i) mask |= (v[i] >= fl ? 1u : 0u) << i;
+            }
+            while (__any_sync(0xffffffffu, mask != 0)) {
+              if (mask != 0) {
+                const int i = __ffs(mask) - 1;
+                mask &= mask - 1;
+                float s = v[0];
+#pragma unroll
+                for (int jj = 1; jj < 32; ++jj) s = (i == jj) ? v[jj] : s;
+                if (s >= list.floor()) list.push(s, static_cast<uint32_t>(id0 + i));
+              }
+            }
           }
         }
       }
@@ -462,6 +477,7 @@ cudaError_t launch_bn(const CUtensorMap& mq, const CUtensorMap& me, const TcPara
                       bool hybrid, cudaStream_t st) {
   switch (list_len_for(prm.k)) {
     case 8: return launch_k<BN, 8>(mq, me, prm, grid, hybrid, st);
+    case 16: return launch_k<BN, 16>(mq, me, prm, grid, hybrid, st);
     case 32: return launch_k<BN, 32>(mq, me, prm, grid, hybrid, st);
     case 128: return launch_k<BN, 128>(mq, me, prm, grid, hybrid, st);
     default: return launch_k<BN, 256>(mq, me, prm, grid, hybrid, st);

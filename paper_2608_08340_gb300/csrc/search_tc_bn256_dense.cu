@@ -8,6 +8,7 @@ cudaError_t launch_bn256_dense(const CUtensorMap& mq, const CUtensorMap& me, con
                                int grid, cudaStream_t st) {
   switch (list_len_for(prm.k)) {
     case 8: return launch_variant<256, 8, false>(mq, me, prm, grid, st);
+    case 16: return launch_variant<256, 16, false>(mq, me, prm, grid, st);
     case 32: return launch_variant<256, 32, false>(mq, me, prm, grid, st);
     case 128: return launch_variant<256, 128, false>(mq, me, prm, grid, st);
     default: return launch_variant<256, 256, false>(mq, me, prm, grid, st);
