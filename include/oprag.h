@@ -172,7 +172,7 @@ OPRAG_API int oprag_index_check(oprag_index *idx);
 
 /* Test hooks: 0 = automatic choice.  OPRAG_OPT_PATH: 1 forces the SIMT
  * streaming kernel, 2 the tensor-core kernel (bf16 only).  OPRAG_OPT_BLOCK_N:
- * corpus rows per tensor-core tile (64 or 256). */
+ * corpus rows per tensor-core tile (128 or 256). */
 #define OPRAG_OPT_PATH 1
 #define OPRAG_OPT_BLOCK_N 2
 OPRAG_API int oprag_index_set_option(oprag_index *idx, int32_t option, int32_t value);

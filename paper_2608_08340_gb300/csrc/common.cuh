@@ -87,47 +87,70 @@ __device__ __forceinline__ void warp_sort_desc(uint64_t (&v)[E]) {
 }
 
 // ---------------------------------------------------------------------------
-// Running top-K of one lane, K <= 32, kept sorted (best first) in registers.
-// Callers test `s >= floor` before push(); floor only ever rises.
+// Running top-K of one lane, K <= 32, kept sorted (best first) in registers as
+// (score, id) pairs.  Candidates must reach a list in increasing id order (the
+// corpus is scanned in id order), so a candidate whose score equals a kept one
+// ranks below it and a strict score compare implements the whole ranking.
+// Empty slots hold (-inf, ~0u); callers test `s > floor` before push().
+constexpr uint32_t kNoId = 0xFFFFFFFFu;
+
 template <int K>
 struct RegTopK {
   static constexpr int kStride = K;     // keys per stored list
-  uint64_t t[K];
+  float s[K];
+  uint32_t id[K];
   float floor;
 
   __device__ __forceinline__ void init() {
 #pragma unroll
-    for (int i = 0; i < K; ++i) t[i] = kEmptyKey;
+    for (int i = 0; i < K; ++i) {
+      s[i] = -INFINITY;
+      id[i] = kNoId;
+    }
     floor = -INFINITY;
   }
 
-  __device__ __forceinline__ void push(float s, uint32_t id) {
-    const uint64_t key = make_key(s, id);
-    if (key > t[K - 1]) {
+  __device__ __forceinline__ bool full() const { return id[K - 1] != kNoId; }
+
+  __device__ __forceinline__ void push(float v, uint32_t vid) {
+    if (v > s[K - 1]) insert(v, vid);
+  }
+
+  // Branch-free insertion; a value not above s[K-1] (e.g. -inf) changes nothing.
+  __device__ __forceinline__ void insert(float v, uint32_t vid) {
 #pragma unroll
-      for (int i = K - 1; i > 0; --i) {
-        const uint64_t prev = t[i - 1];
-        t[i] = key > prev ? prev : (key > t[i] ? key : t[i]);
-      }
-      t[0] = umax64(t[0], key);
-      floor = key_floor(t[K - 1]);
+    for (int i = K - 1; i > 0; --i) {
+      const bool above_prev = v > s[i - 1];
+      const bool above_here = v > s[i];
+      s[i] = above_prev ? s[i - 1] : (above_here ? v : s[i]);
+      id[i] = above_prev ? id[i - 1] : (above_here ? vid : id[i]);
     }
+    const bool top = v > s[0];
+    s[0] = top ? v : s[0];
+    id[0] = top ? vid : id[0];
+    floor = s[K - 1];
+  }
+
+  __device__ __forceinline__ uint64_t key(int i) const {
+    return id[i] == kNoId ? kEmptyKey : make_key(s[i], id[i]);
   }
 
   __device__ __forceinline__ void store(uint64_t* dst) const {
 #pragma unroll
     for (int i = 0; i < K; i += 2)
-      *reinterpret_cast<ulonglong2*>(dst + i) = make_ulonglong2(t[i], t[i + 1]);
+      *reinterpret_cast<ulonglong2*>(dst + i) = make_ulonglong2(key(i), key(i + 1));
   }
 
   __device__ __forceinline__ void load(const uint64_t* src) {
 #pragma unroll
     for (int i = 0; i < K; i += 2) {
       const ulonglong2 v = *reinterpret_cast<const ulonglong2*>(src + i);
-      t[i] = v.x;
-      t[i + 1] = v.y;
+      s[i] = key_floor(v.x);
+      id[i] = v.x == kEmptyKey ? kNoId : key_id(v.x);
+      s[i + 1] = key_floor(v.y);
+      id[i + 1] = v.y == kEmptyKey ? kNoId : key_id(v.y);
     }
-    floor = key_floor(t[K - 1]);
+    floor = s[K - 1];
   }
 };
 

@@ -24,6 +24,11 @@ struct ListSet {
   int P;
   int TH;
   int stride;
+  // Tensor-core lists: only producers p < sets * (C - first_cta(tile)) exist
+  // for a tile (see search_tc.cuh); C == 0 means all P lists exist.
+  int C = 0;
+  int qt = 0;
+  int sets = 1;
 };
 
 // Optional lexical part of the fused score (Sec. 4.4 weighted fusion):
@@ -52,11 +57,12 @@ cudaError_t launch_simt_search(int dtype, const void* E, const void* Q, const Se
 
 // --- tcgen05 tensor-core search (bf16).
 struct TcPlan {
-  int block_n;     // corpus rows per tile: 64, 128 or 256
+  int block_n;     // corpus rows per tile: 128 or 256
   int grid;        // CTAs (persistent)
   int qt;          // query tiles of 128
-  int slots;       // query tiles visited per CTA
-  int P;           // lists per query tile
+  int nt;          // corpus tiles
+  int win;         // corpus tiles per L2 window
+  int pmax;        // lists per query tile
   int stages;
   size_t smem;
 };

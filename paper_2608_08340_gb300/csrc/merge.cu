@@ -42,7 +42,13 @@ merge_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
   const int tile = qi / ls.TH, row = qi % ls.TH;
   const uint64_t* base = ls.keys + (static_cast<int64_t>(tile) * ls.P * ls.TH + row) * ls.stride;
   const int64_t list_step = static_cast<int64_t>(ls.TH) * ls.stride;
-  const int total = ls.P * k;
+  int np = ls.P;
+  if (ls.C > 0) {
+    int c0 = static_cast<int>(static_cast<int64_t>(tile) * ls.C / ls.qt) - 1;
+    c0 = c0 < 0 ? 0 : c0;
+    np = min(ls.P, (ls.C - c0) * ls.sets);
+  }
+  const int total = np * k;
   const int lo = static_cast<int>(static_cast<int64_t>(total) * warp / kMergeWarps);
   const int hi = static_cast<int>(static_cast<int64_t>(total) * (warp + 1) / kMergeWarps);
 

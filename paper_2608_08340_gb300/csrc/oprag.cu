@@ -607,7 +607,7 @@ int oprag_index_set_option(oprag_index* idx, int32_t option, int32_t value) {
     return ok();
   }
   if (option == OPRAG_OPT_BLOCK_N) {
-    if (value != 0 && value != 64 && value != 256)
+    if (value != 0 && value != 128 && value != 256)
       return fail(OPRAG_ERR_INVALID_ARG, "block_n %d", value);
     idx->opt_block_n = value;
     return ok();

@@ -1,5 +1,9 @@
 // Host planning for the tensor-core search kernel of search_tc.cuh: tile
-// size, persistent grid, slot bookkeeping, scratch size and TMA descriptors.
+// size, persistent grid, window size and list bound, scratch size and TMA
+// descriptors.
+#include <algorithm>
+#include <vector>
+
 #include "search_tc.cuh"
 
 namespace oprag {
@@ -43,46 +47,63 @@ bool make_map(CUtensorMap* m, const void* base, int64_t rows, int d, int box_row
          CUDA_SUCCESS;
 }
 
-int gcd_int(int a, int b) {
-  while (b) {
-    const int t = a % b;
-    a = b;
-    b = t;
-  }
-  return a;
-}
-
 }  // namespace
 
 TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n) {
   TcPlan pl{};
   pl.qt = (s.q + kBlockM - 1) / kBlockM;
   int bn = 256;
-  if (force_block_n == 64 || force_block_n == 256) {
+  if (force_block_n == 128 || force_block_n == 256) {
     bn = force_block_n;
   } else {
-    // Small query batches leave few units: cut the corpus finer so that every
-    // SM gets several units.
+    // Few units (small query batches): 128-row tiles give every SM more of
+    // them; the MMA rate per row is the same for N = 128 and N = 256.
     const int64_t units256 = static_cast<int64_t>(pl.qt) * ((s.n + 255) / 256);
-    if (units256 < 4LL * num_sms) bn = 64;
+    if (units256 < 4LL * num_sms) bn = 128;
   }
   pl.block_n = bn;
-  const int64_t nt = (s.n + bn - 1) / bn;
-  const int64_t units = nt * pl.qt;
+  pl.nt = static_cast<int>((s.n + bn - 1) / bn);
+  const int64_t units = static_cast<int64_t>(pl.nt) * pl.qt;
   pl.grid = static_cast<int>(units < num_sms ? units : num_sms);
   if (pl.grid < 1) pl.grid = 1;
-  const int g = gcd_int(pl.grid, pl.qt);
-  pl.slots = pl.qt / g;
-  pl.P = pl.grid / g;
-  pl.stages = bn == 64 ? stages_for<64>() : stages_for<256>();
-  pl.smem = bn == 64 ? smem_for<64>() : smem_for<256>();
+  // Windows of about 32 MB of corpus (one window when the corpus is small).
+  const int64_t tile_bytes = static_cast<int64_t>(bn) * s.d * 2;
+  const int64_t corpus = tile_bytes * pl.nt;
+  pl.win = corpus <= (int64_t(80) << 20)
+               ? pl.nt
+               : static_cast<int>(std::max<int64_t>(1, (int64_t(32) << 20) / tile_bytes));
+  // Exact per-tile range of CTAs, by replaying the schedule of UnitSeq.
+  const int C = pl.grid;
+  int per_tile = 1;
+  std::vector<int> hi(pl.qt, -1);
+  bool ok = true;
+  for (int w = 0; static_cast<int64_t>(w) * pl.win < pl.nt; ++w) {
+    const int tw = std::min(pl.win, pl.nt - w * pl.win);
+    const int64_t uw = static_cast<int64_t>(pl.qt) * tw;
+    for (int c = 0; c < C; ++c) {
+      const int64_t l0 = uw * c / C, l1 = uw * (c + 1) / C;
+      if (l0 >= l1) continue;
+      for (int64_t j = l0 / tw; j <= (l1 - 1) / tw; ++j) {
+        if (c < first_cta(static_cast<int>(j), pl.qt, C)) ok = false;
+        hi[j] = std::max(hi[j], c);
+      }
+    }
+  }
+  for (int j = 0; j < pl.qt; ++j)
+    per_tile = std::max(per_tile, hi[j] - first_cta(j, pl.qt, C) + 1);
+  if (!ok) per_tile = C;  // not expected; every CTA then gets a slot per tile
+  pl.pmax = per_tile * epi_sets(list_len_for(s.k));
+  pl.stages = bn == 128 ? stages_for<128>() : stages_for<256>();
+  const int K = list_len_for(s.k);
+  pl.smem = bn == 128 ? (K <= 16 ? smem_for<128, 16>() : smem_for<128, 32>())
+                      : (K <= 16 ? smem_for<256, 16>() : smem_for<256, 32>());
   return pl;
 }
 
 size_t tc_scratch_bytes(const SearchShape& s, const TcPlan& pl) {
   const int K = list_len_for(s.k);
   const int stride = K > 32 ? 2 * K : K;
-  const size_t rows = static_cast<size_t>(pl.qt) * pl.P * kBlockM;
+  const size_t rows = static_cast<size_t>(pl.qt) * pl.pmax * kBlockM;
   size_t bytes = rows * stride * sizeof(uint64_t);
   if (K > 32) bytes += rows * (sizeof(uint64_t) + sizeof(int));
   return bytes;
@@ -96,17 +117,16 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
     return cudaErrorInvalidValue;
   const int K = list_len_for(s.k);
   const int stride = K > 32 ? 2 * K : K;
-  const size_t rows = static_cast<size_t>(pl.qt) * pl.P * kBlockM;
+  const size_t rows = static_cast<size_t>(pl.qt) * pl.pmax * kBlockM;
   TcParams prm{};
   prm.n = s.n;
   prm.d = s.d;
   prm.q = s.q;
   prm.k = s.k;
   prm.qt = pl.qt;
-  prm.units = static_cast<int64_t>(pl.qt) * ((s.n + pl.block_n - 1) / pl.block_n);
-  prm.g = gcd_int(pl.grid, pl.qt);
-  prm.P = pl.P;
-  prm.slots = pl.slots;
+  prm.nt = pl.nt;
+  prm.win = pl.win;
+  prm.pmax = pl.pmax;
   prm.kblocks = (s.d + kBlockK - 1) / kBlockK;
   prm.fu = fu;
   prm.lists = static_cast<uint64_t*>(scratch);
@@ -114,11 +134,14 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
   prm.meta_count = reinterpret_cast<int*>(prm.meta_worst + (K > 32 ? rows : 0));
   prm.dev_err = dev_err;
   lists->keys = prm.lists;
-  lists->P = pl.P;
+  lists->P = pl.pmax;
   lists->TH = kBlockM;
   lists->stride = stride;
+  lists->C = pl.grid;
+  lists->qt = pl.qt;
+  lists->sets = epi_sets(K);
   const bool hybrid = fu.bm25 != nullptr;
-  if (pl.block_n == 64) return launch_bn64(mq, me, prm, pl.grid, hybrid, st);
+  if (pl.block_n == 128) return launch_bn128(mq, me, prm, pl.grid, hybrid, st);
   return hybrid ? launch_bn256_fused(mq, me, prm, pl.grid, st)
                 : launch_bn256_dense(mq, me, prm, pl.grid, st);
 }

@@ -14,17 +14,18 @@
 // running top-K list per query for each of them ("slots") and leaves it as
 // partial list p = c / g of tile j for the merge kernel.
 //
-// Roles (192 threads):
+// Roles (320 threads):
 //   warp 0, lane 0: TMA producer.  Per K block of 64 bf16 (one 128-byte
 //                   swizzle row) it loads the 128 x 64 query tile and the
 //                   BN x 64 corpus tile into a pipeline stage.
 //   warp 1        : allocates 2 x BN TMEM columns (two fp32 accumulators);
 //                   lane 0 issues tcgen05.mma (M = 128, N = BN, K = 16).
-//   warps 2..5    : epilogue.  Each thread owns one query (one TMEM lane),
-//                   reads its BN scores with tcgen05.ld and filters them
-//                   against its running k-th best score.
-// The two accumulators let the epilogue of one unit overlap the MMAs of the
-// next.  Every mbarrier wait is bounded (see common.cuh).
+//   warps 2..9    : epilogue, two sets of four warps, set s draining
+//                   accumulator s.  Each thread owns one query (one TMEM
+//                   lane), reads its BN scores with tcgen05.ld and filters
+//                   them against its running k-th best score.
+// The two accumulators let the MMAs of one unit overlap the filtering of the
+// previous two.  Every mbarrier wait is bounded (see common.cuh).
 #pragma once
 #include <cuda.h>
 
@@ -37,7 +38,11 @@ namespace tc {
 constexpr int kBlockM = 128;
 constexpr int kBlockK = 64;                 // bf16 per 128-byte row
 constexpr int kUmmaK = 16;
-constexpr int kThreads = 192;
+// Epilogue warp sets: two (one per accumulator, 320 threads) for register
+// lists up to 16 keys; one set (192 threads, more registers per thread) for
+// the longer lists.
+__host__ __device__ constexpr int epi_sets(int K) { return K <= 16 ? 2 : 1; }
+__host__ __device__ constexpr int threads_for(int K) { return 64 + 128 * epi_sets(K); }
 constexpr uint32_t kAStageBytes = kBlockM * kBlockK * 2;
 constexpr int kSmemBudget = 200 * 1024;
 
@@ -46,27 +51,80 @@ struct TcParams {
   int d;
   int q;
   int k;
-  int qt;
-  int64_t units;
-  int g;
-  int P;
-  int slots;
+  int qt;               // query tiles of 128
+  int nt;               // corpus tiles of BN rows
+  int win;              // corpus tiles per L2 window
+  int pmax;             // lists per query tile (CTAs that may touch it x kEpiSets)
   int kblocks;
   Fusion fu;
-  uint64_t* lists;      // [(j * P + p) * 128 + row] * stride
+  uint64_t* lists;      // [(j * pmax + producer) * 128 + row] * stride
   int* meta_count;      // buffered lists: kept keys per (list, row)
   uint64_t* meta_worst; // buffered lists: K-th key per (list, row)
   int* dev_err;
 };
+
+// Units of one CTA in processing order.  The corpus tiles are cut into
+// windows of `win` tiles (sized to stay in L2); inside a window the units
+// (query tile j, corpus tile t) are ordered j-major and split into C equal
+// contiguous shares, share c going to CTA c.  So all CTAs sweep the windows
+// together (each window is read from HBM once and re-read from L2), while a
+// CTA meets only the one or two query tiles its share covers and scans their
+// corpus tiles in increasing order.
+struct UnitSeq {
+  int nt, win, qt, C, cta;
+  int w, tw;
+  int64_t l, l_end;
+
+  __device__ __forceinline__ void start(const TcParams& p, int cta_, int C_) {
+    nt = p.nt;
+    win = p.win;
+    qt = p.qt;
+    C = C_;
+    cta = cta_;
+    w = -1;
+    next_window();
+  }
+  __device__ __forceinline__ void next_window() {
+    while (true) {
+      ++w;
+      if (static_cast<int64_t>(w) * win >= nt) {
+        l = l_end = 0;
+        return;
+      }
+      tw = min(win, nt - w * win);
+      const int64_t uw = static_cast<int64_t>(qt) * tw;
+      l = uw * cta / C;
+      l_end = uw * (cta + 1) / C;
+      if (l < l_end) return;
+    }
+  }
+  __device__ __forceinline__ bool valid() const { return static_cast<int64_t>(w) * win < nt; }
+  __device__ __forceinline__ void next() {
+    if (++l >= l_end) next_window();
+  }
+  __device__ __forceinline__ int j() const { return static_cast<int>(l / tw); }
+  __device__ __forceinline__ int t() const { return w * win + static_cast<int>(l % tw); }
+};
+
+// First CTA whose shares can reach query tile j (the host checks the bound).
+__host__ __device__ __forceinline__ int first_cta(int j, int qt, int C) {
+  const int c = static_cast<int>(static_cast<int64_t>(j) * C / qt) - 1;
+  return c < 0 ? 0 : c;
+}
 
 template <int BN>
 constexpr int stages_for() {
   return kSmemBudget / (kAStageBytes + BN * 128) > 8 ? 8 : kSmemBudget / (kAStageBytes + BN * 128);
 }
 
-template <int BN>
+// Per epilogue thread: one 32-float row where a chunk's scores are staged so
+// that candidate columns can be read back by index.
+constexpr int kStageRowBytes = 32 * 4;
+
+template <int BN, int K>
 constexpr size_t smem_for() {
-  return static_cast<size_t>(stages_for<BN>()) * (kAStageBytes + BN * 128) + 1024 + 256;
+  return static_cast<size_t>(stages_for<BN>()) * (kAStageBytes + BN * 128) +
+         static_cast<size_t>(epi_sets(K)) * 128 * kStageRowBytes + 1024 + 256;
 }
 
 // ----------------------------------------------------------------- PTX
@@ -140,8 +198,9 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar) {
       : "memory");
 }
 
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
-  uint32_t r[32];
+// Issues a 32-column TMEM load (32 lanes x 32 columns of 32 bits); the
+// registers are valid only after tmem_wait_ld() on the same array.
+__device__ __forceinline__ void tmem_ld32_async(uint32_t taddr, uint32_t (&r)[32]) {
   asm volatile(
       "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
       "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
@@ -152,9 +211,32 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
         "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
         "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
       : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Waits for the outstanding TMEM loads.  The registers are passed through the
+// asm so that no use of them can be scheduled before the wait.
+__device__ __forceinline__ void tmem_wait_ld(uint32_t (&r)[32]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]),
+                 "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]),
+                 "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]),
+                 "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]),
+                 "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]),
+                 "+r"(r[30]), "+r"(r[31])
+               :
+               : "memory");
+}
+
+// max of 32 values, depth-5 tree.
+__device__ __forceinline__ float max32(const float (&v)[32]) {
+  float a[16];
 #pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+  for (int i = 0; i < 16; ++i) a[i] = fmaxf(v[2 * i], v[2 * i + 1]);
+#pragma unroll
+  for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+    for (int i = 0; i < w; ++i) a[i] = fmaxf(a[2 * i], a[2 * i + 1]);
+  return a[0];
 }
 
 // Waits without looking at the abort word (used to drain in-flight copies and
@@ -187,8 +269,10 @@ struct EpiList<K, false> {
   __device__ __forceinline__ void load(const TcParams& p, int64_t sr) { t.load(p.lists + sr * K); }
   __device__ __forceinline__ void save(const TcParams& p, int64_t sr) { t.store(p.lists + sr * K); }
   __device__ __forceinline__ void clear() { t.init(); }
+  __device__ __forceinline__ bool full() const { return t.full(); }
   __device__ __forceinline__ float floor() const { return t.floor; }
   __device__ __forceinline__ void push(float s, uint32_t id) { t.push(s, id); }
+  __device__ __forceinline__ void insert(float s, uint32_t id) { t.insert(s, id); }
   __device__ __forceinline__ void sync(bool, bool) {}
   __device__ __forceinline__ void finalize(const TcParams&, int64_t, bool) {}
 };
@@ -217,8 +301,12 @@ struct EpiList<K, true> {
     t.worst = kEmptyKey;
     t.floor = -INFINITY;
   }
+  __device__ __forceinline__ bool full() const { return t.worst != kEmptyKey; }
   __device__ __forceinline__ float floor() const { return t.floor; }
   __device__ __forceinline__ void push(float s, uint32_t id) { t.push(s, id); }
+  __device__ __forceinline__ void insert(float s, uint32_t id) {
+    if (s > -INFINITY) t.push(s, id);
+  }
   __device__ __forceinline__ void sync(bool final, bool active) { t.sync(final, active); }
   // Warp-collective: sorts the lane's buffer, best K first.
   __device__ __forceinline__ void finalize(const TcParams& p, int64_t sr, bool valid) {
@@ -230,18 +318,20 @@ struct EpiList<K, true> {
 // ----------------------------------------------------------------- kernel
 
 template <int BN, int K, bool kHybrid>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(threads_for(K), 1)
 tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_e,
                  const TcParams p) {
   constexpr int S = stages_for<BN>();
   constexpr uint32_t kBStageBytes = BN * 128;
   constexpr uint32_t kTmemCols = 2 * BN;
+  constexpr int kEpiSets = epi_sets(K);
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* base = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   unsigned char* sA = base;
   unsigned char* sB = sA + S * kAStageBytes;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sB + S * kBStageBytes);
+  float* stage_rows = reinterpret_cast<float*>(sB + S * kBStageBytes);   // epilogue staging
+  uint64_t* full = reinterpret_cast<uint64_t*>(stage_rows + kEpiSets * 128 * 32);
   uint64_t* empty = full + S;
   uint64_t* tfull = empty + S;
   uint64_t* tempty = tfull + 2;
@@ -280,9 +370,10 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       uint32_t ph = 0;
       uint32_t issued = 0, parity = 0;    // per stage: ever issued, parity of last issue
       bool ok = true;
-      for (int64_t u = cta; ok && u < p.units; u += C) {
-        const int j = static_cast<int>(u % p.qt);
-        const int t = static_cast<int>(u / p.qt);
+      UnitSeq us;
+      for (us.start(p, cta, C); ok && us.valid(); us.next()) {
+        const int j = us.j();
+        const int t = us.t();
         for (int kb = 0; kb < p.kblocks; ++kb) {
           if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, p.dev_err)) { ok = false; break; }
           mbar_arrive_expect_tx(&full[s], kAStageBytes + kBStageBytes);
@@ -306,7 +397,8 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       int acc = 0;
       uint32_t acc_ph = 0;
       bool ok = true;
-      for (int64_t u = cta; ok && u < p.units; u += C) {
+      UnitSeq us;
+      for (us.start(p, cta, C); ok && us.valid(); us.next()) {
         if (!mbar_wait(&tempty[acc], acc_ph ^ 1u, abort_flag, p.dev_err)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
@@ -331,54 +423,76 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     __syncwarp();
   } else {
     // ------------------------------------------------ epilogue
+    // kEpiSets sets of four warps; set s filters the units whose sequence
+    // number is s modulo kEpiSets (with two sets, two units are filtered at
+    // the same time).  Each set keeps its own lists.
+    const int set = (warp - 2) >> 2;
     const int eg = warp & 3;                 // TMEM lane group of this warp
     const int row = eg * 32 + lane;          // query row within a tile
-    const int c_mod = cta % p.g, my_p = cta / p.g;
+    const int per_tile = p.pmax / kEpiSets;  // CTAs per query tile with a list slot
+    auto list_row = [&](int j) -> int64_t {
+      const int pc = cta - first_cta(j, p.qt, C);
+      return (static_cast<int64_t>(j) * p.pmax + pc * kEpiSets + set) * kBlockM + row;
+    };
+    auto owns = [&](int j) {
+      const int pc = cta - first_cta(j, p.qt, C);
+      return pc >= 0 && pc < per_tile;
+    };
     EpiList<K> list;
     list.clear();
 
-    for (int s = 0; s < p.slots; ++s) {
-      const int j = c_mod + s * p.g;
-      if (j * kBlockM + row < p.q) list.init_mem(p, (static_cast<int64_t>(j) * p.P + my_p) * kBlockM + row);
-    }
+    // This CTA owns the list slots (j, cta - first_cta(j)); empty them first.
+    for (int j = 0; j < p.qt; ++j)
+      if (owns(j) && j * kBlockM + row < p.q) list.init_mem(p, list_row(j));
 
-    int cur_slot = -1;
+    int cur_j = -1;
     int64_t cur_sr = 0;
     bool cur_valid = false;
-    int acc = 0;
-    uint32_t acc_ph = 0;
-    for (int64_t u = cta; u < p.units; u += C) {
-      const int j = static_cast<int>(u % p.qt);
-      const int64_t t = u / p.qt;
-      const int slot = (j - c_mod) / p.g;
+    uint32_t acc_ph = 0;                     // phase bit per accumulator
+    UnitSeq us;
+    int seq = 0;
+    for (us.start(p, cta, C); us.valid(); us.next(), ++seq) {
+      if (seq % kEpiSets != set) continue;
+      const int acc = seq & 1;
+      const int j = us.j();
+      const int64_t t = us.t();
       const bool valid = j * kBlockM + row < p.q;
       const bool warp_live = j * kBlockM + eg * 32 < p.q;
-      if (slot != cur_slot) {
-        if (cur_slot >= 0 && cur_valid) list.save(p, cur_sr);
-        cur_slot = slot;
-        cur_sr = (static_cast<int64_t>(j) * p.P + my_p) * kBlockM + row;
-        cur_valid = valid;
-        if (valid) list.load(p, cur_sr); else list.clear();
+      if (j != cur_j) {
+        if (cur_j >= 0 && cur_valid) list.save(p, cur_sr);
+        if (!owns(j)) {              // cannot happen when the host plan holds
+          atomicExch(p.dev_err, 2);
+          *abort_flag = 1;
+        }
+        cur_j = j;
+        cur_sr = list_row(j);
+        cur_valid = valid && owns(j);
+        if (cur_valid) list.load(p, cur_sr); else list.clear();
       }
-      if (!mbar_wait(&tfull[acc], acc_ph, abort_flag, p.dev_err)) break;
+      const bool act = cur_valid;
+      if (!mbar_wait(&tfull[acc], (acc_ph >> acc) & 1u, abort_flag, p.dev_err)) break;
       tc_fence_after();
       if (warp_live) {
         float inv_max = 0.f;
         const float* brow = nullptr;
-        if (kHybrid && valid) {
+        if (kHybrid && act) {
           const float m = p.fu.bm25_max[j * kBlockM + row];
           inv_max = m > 0.f ? 1.f / m : 0.f;
           brow = p.fu.bm25 + static_cast<int64_t>(j * kBlockM + row) * p.fu.ld;
         }
         const uint32_t taddr = tmem_base + (static_cast<uint32_t>(eg * 32) << 16) +
                                static_cast<uint32_t>(acc * BN);
-#pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
-          float v[32];
-          __syncwarp();
-          tmem_ld32(taddr + c * 32, v);
+        // This thread's staging row; float4 groups are XOR-swizzled by lane so
+        // that the 32 lanes' 16-byte stores spread over all banks.
+        float* srow = stage_rows + ((warp - 2) * 32 + lane) * 32;
+        const int swz = lane & 7;
+        // Scores of one chunk (corpus rows id0 .. id0 + 31), fused with the
+        // lexical part when hybrid, -inf past the end of the corpus.
+        auto scores = [&](const uint32_t (&r)[32], int c, float (&v)[32]) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
           const int64_t id0 = t * BN + c * 32;
-          if (kHybrid && valid) {
+          if (kHybrid && act) {
             const float a = p.fu.alpha, b1 = 1.f - p.fu.alpha;
             if (id0 + 32 <= p.n) {
 #pragma unroll
@@ -400,44 +514,95 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             for (int i = 0; i < 32; ++i)
               if (id0 + i >= p.n) v[i] = -INFINITY;
           }
-          list.sync(false, valid);
-          float m = v[0];
-#pragma unroll
-          for (int i = 1; i < 32; ++i) m = fmaxf(m, v[i]);
-          const float fl = list.floor();
-          if (__any_sync(0xffffffffu, valid && m >= fl)) {
+        };
+        // Filters one chunk against max(list floor, unit bound).
+        auto process = [&](const uint32_t (&r)[32], int c, float bound) {
+          float v[32];
+          scores(r, c, v);
+          const int64_t id0 = t * BN + c * 32;
+          list.sync(false, act);
+          const float fl = fmaxf(list.floor(), bound);
+          if (__any_sync(0xffffffffu, act && max32(v) >= fl)) {
             // Lanes insert their candidates together, one column per round,
             // so the warp runs max-per-lane rounds instead of the sum.
             uint32_t mask = 0;
-            if (valid) {
+            if (act) {
 #pragma unroll
               for (int i = 0; i < 32; ++i) mask |= (v[i] >= fl ? 1u : 0u) << i;
-            }
-            while (__any_sync(0xffffffffu, mask != 0)) {
-              if (mask != 0) {
-                const int i = __ffs(mask) - 1;
-                mask &= mask - 1;
-                float s = v[0];
 #pragma unroll
-                for (int jj = 1; jj < 32; ++jj) s = (i == jj) ? v[jj] : s;
-                if (s >= list.floor()) list.push(s, static_cast<uint32_t>(id0 + i));
-              }
+              for (int g = 0; g < 8; ++g)
+                *reinterpret_cast<float4*>(srow + ((g ^ swz) << 2)) =
+                    make_float4(v[4 * g], v[4 * g + 1], v[4 * g + 2], v[4 * g + 3]);
+            }
+            // Warp-uniform number of rounds; each round takes the lowest
+            // remaining candidate column of every lane (ids stay increasing)
+            // and inserts it with the branch-free network, so rounds are
+            // straight-line code and the next extraction overlaps the insert.
+            const int rounds = __reduce_max_sync(0xffffffffu, __popc(mask));
+#pragma unroll 2
+            for (int r = 0; r < rounds; ++r) {
+              const int i = __ffs(mask) - 1;
+              const bool has = mask != 0;
+              mask &= mask - 1;
+              const float s = has ? srow[((((i & 31) >> 2) ^ swz) << 2) | (i & 3)] : -INFINITY;
+              list.insert(s, static_cast<uint32_t>(id0 + i));
             }
           }
+          __syncwarp();
+        };
+        constexpr int NC = BN / 32;
+        static_assert(NC % 2 == 0, "chunks are processed in pairs");
+        uint32_t ra[32], rb[32];
+        float bound = -INFINITY;
+        if constexpr (K <= 32) {
+          if (__any_sync(0xffffffffu, act && !list.full())) {
+          // A list that is not full yet would take almost every score of this
+          // unit as a candidate.  Cut the unit into K groups of BN / K
+          // scores: each group holds a score >= its maximum, so the smallest
+          // group maximum is <= the unit's K-th best score and nothing below
+          // it can enter the list.
+          constexpr int G = K / NC;           // groups per chunk
+          static_assert(G >= 1 && 32 % G == 0, "group layout");
+          float gmin = INFINITY;
+#pragma unroll 1
+          for (int c = 0; c < NC; ++c) {
+            __syncwarp();
+            tmem_ld32_async(taddr + c * 32, ra);
+            tmem_wait_ld(ra);
+            float v[32];
+            scores(ra, c, v);
+#pragma unroll
+            for (int g = 0; g < G; ++g) {
+              float m = v[g * (32 / G)];
+#pragma unroll
+              for (int i = 1; i < 32 / G; ++i) m = fmaxf(m, v[g * (32 / G) + i]);
+              gmin = fminf(gmin, m);
+            }
+          }
+          bound = gmin;
+          }
+        }
+        __syncwarp();
+        tmem_ld32_async(taddr, ra);
+#pragma unroll 1
+        for (int c = 0; c < NC; c += 2) {
+          tmem_wait_ld(ra);
+          tmem_ld32_async(taddr + (c + 1) * 32, rb);
+          process(ra, c, bound);
+          tmem_wait_ld(rb);
+          if (c + 2 < NC) tmem_ld32_async(taddr + (c + 2) * 32, ra);
+          process(rb, c + 1, bound);
         }
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);
-      if (++acc == 2) { acc = 0; acc_ph ^= 1u; }
+      acc_ph ^= 1u << acc;
     }
-    if (cur_slot >= 0 && cur_valid) list.save(p, cur_sr);
+    if (cur_j >= 0 && cur_valid) list.save(p, cur_sr);
     if (K > 32) {
-      for (int s = 0; s < p.slots; ++s) {
-        const int j = c_mod + s * p.g;
-        const bool valid = j * kBlockM + row < p.q;
-        list.finalize(p, (static_cast<int64_t>(j) * p.P + my_p) * kBlockM + row, valid);
-      }
+      for (int j = 0; j < p.qt; ++j)
+        if (owns(j)) list.finalize(p, list_row(j), j * kBlockM + row < p.q);
     }
   }
 
@@ -452,7 +617,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
 template <int BN, int K, bool H>
 cudaError_t launch_variant(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
                            int grid, cudaStream_t st) {
-  constexpr size_t smem = smem_for<BN>();
+  constexpr size_t smem = smem_for<BN, K>();
   static bool configured = false;
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(tc_search_kernel<BN, K, H>,
@@ -461,7 +626,7 @@ cudaError_t launch_variant(const CUtensorMap& mq, const CUtensorMap& me, const T
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  tc_search_kernel<BN, K, H><<<grid, kThreads, smem, st>>>(mq, me, prm);
+  tc_search_kernel<BN, K, H><<<grid, threads_for(K), smem, st>>>(mq, me, prm);
   return cudaGetLastError();
 }
 
@@ -485,7 +650,7 @@ cudaError_t launch_bn(const CUtensorMap& mq, const CUtensorMap& me, const TcPara
 }
 
 // Instantiations live in their own translation units (parallel builds).
-cudaError_t launch_bn64(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm, int grid,
+cudaError_t launch_bn128(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm, int grid,
                         bool hybrid, cudaStream_t st);
 cudaError_t launch_bn256_dense(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
                                int grid, cudaStream_t st);

@@ -89,7 +89,7 @@ def test_ragged_shapes(n, d, q, k, path):
     check_dense(ids, sc, E, Q, k, f"ragged n={n} d={d} q={q} k={k} {path}")
 
 
-@pytest.mark.parametrize("bn", [64, 256])
+@pytest.mark.parametrize("bn", [128, 256])
 def test_tc_tile_widths_agree(bn):
     w = workloads.config(1, n=9000, batch=300)
     idx = _index(w.E_data)
