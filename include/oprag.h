@@ -196,6 +196,32 @@ OPRAG_API int oprag_index_last_timing(oprag_index *idx, float *lexical_ms, float
  * core, 0 none yet. */
 OPRAG_API int oprag_index_last_path(const oprag_index *idx);
 
+/*
+ * oprag_search without any device allocation.  The paper has no counterpart:
+ * this entry point serves callers that must not allocate device memory while
+ * answering a request -- a serving process whose memory pool has already
+ * claimed the GPU, or a host that cannot afford the device-wide
+ * synchronisation that cudaMalloc / cudaFree may cause.
+ *
+ * Same arguments, results and stream semantics as oprag_search.  Instead of
+ * the index's scratch buffer (which oprag_search grows with cudaMalloc), the
+ * partial top-k lists live in one statically sized device array of 16 MiB
+ * that the library holds on every GPU that loads it until the process exits.
+ *   - A search whose lists need more than 16 MiB (many queries with a large
+ *     k, e.g. k > 32 over thousands of queries) is refused with
+ *     OPRAG_ERR_INVALID_ARG and a message giving the required size; nothing
+ *     is launched.
+ *   - The first call on a device resolves the array's device address (a
+ *     runtime query, no allocation); make that first call before any stream
+ *     capture.
+ *   - All calls share the array, so calls that overlap on the GPU (different
+ *     indexes or streams without ordering between them) race; order them.
+ *     The kernels initialise every list they use, so nothing from an earlier
+ *     call leaks into a later one.
+ */
+OPRAG_API int oprag_search_noalloc(oprag_index *idx, const void *queries, int32_t q, int32_t k,
+                                   int64_t *out_ids, float *out_scores, void *stream);
+
 /* Message of the last failed call on this thread ("" if none). */
 OPRAG_API const char *oprag_last_error(void);
 

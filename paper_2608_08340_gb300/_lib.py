@@ -42,6 +42,7 @@ SIGNATURES = {
     "oprag_upsert": (_I32, [_P, _P, _P, _I64, _I32, _I32, _P]),
     "oprag_search": (_I32, [_P, _P, _I32, _I32, _P, _P, _P]),
     "oprag_search_host": (_I32, [_P, _P, _I32, _I32, _P, _P, _P]),
+    "oprag_search_noalloc": (_I32, [_P, _P, _I32, _I32, _P, _P, _P]),
     "oprag_index_set_sparse": (_I32, [_P, _P, _P, _I32, _F, _F]),
     "oprag_hybrid_search": (_I32, [_P, _P, _I32, _P, _P, _F, _I32, _P, _P, _P]),
     "oprag_index_check": (_I32, [_P]),

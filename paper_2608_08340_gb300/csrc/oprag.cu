@@ -5,6 +5,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <string>
 #include <unordered_set>
 #include <vector>
@@ -636,3 +637,81 @@ int oprag_index_last_timing(oprag_index* idx, float* lexical_ms, float* search_m
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Search without device allocations.  The partial lists live in a statically
+// sized device array instead of the index's lazily grown scratch buffer.  The
+// paper has no counterpart; this serves callers that must not allocate device
+// memory while serving a request.
+
+namespace {
+
+constexpr size_t kStaticScratchBytes = size_t(16) << 20;
+constexpr int kMaxDevices = 64;
+
+}  // namespace
+
+// Shared by every call on a device; kept until the process exits.
+static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+
+namespace {
+
+std::mutex g_static_mu;
+void* g_static_ptr[kMaxDevices] = {};
+
+// Device address of g_static_scratch on `device` (which must be current),
+// resolved once per device.  The host-side name is only a stand-in.
+int static_scratch(int device, void** out) {
+  if (device < 0 || device >= kMaxDevices)
+    return fail(OPRAG_ERR_INVALID_ARG, "device %d out of range", device);
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (g_static_ptr[device] == nullptr) {
+    void* ptr = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&ptr, g_static_scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "resolving the static scratch array");
+    g_static_ptr[device] = ptr;
+  }
+  *out = g_static_ptr[device];
+  return OPRAG_OK;
+}
+
+}  // namespace
+
+extern "C" int oprag_search_noalloc(oprag_index* idx, const void* queries, int32_t q, int32_t k,
+                                    int64_t* out_ids, float* out_scores, void* stream) {
+  int rc = check_search_args(idx, queries, q, k, out_ids, out_scores);
+  if (rc) return rc;
+  if (q == 0) return ok();
+  DeviceGuard g(idx->device);
+  void* scratch = nullptr;
+  if ((rc = static_scratch(idx->device, &scratch))) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  SearchShape s{idx->n, idx->d, q, k};
+  const int path = choose_path(idx, q);
+  size_t need;
+  TcPlan plan{};
+  int grid = 0;
+  if (path == 1) {
+    grid = simt_grid(s, idx->num_sms);
+    need = simt_scratch_bytes(idx->dtype, s, grid);
+  } else {
+    plan = tc_plan(s, idx->num_sms, idx->opt_block_n);
+    need = tc_scratch_bytes(s, plan);
+  }
+  if (need > kStaticScratchBytes)
+    return fail(OPRAG_ERR_INVALID_ARG,
+                "this search needs %zu bytes of scratch but the static array holds %zu; use "
+                "oprag_search or fewer queries / a smaller k",
+                need, kStaticScratchBytes);
+  if ((rc = begin_call(idx, st))) return rc;
+  const Fusion none{nullptr, 0, nullptr, 0.f};
+  ListSet lists{};
+  cudaError_t e =
+      path == 1 ? launch_simt_search(idx->dtype, idx->emb, queries, s, none, scratch, grid, &lists, st)
+                : launch_tc_search(idx->emb, queries, s, none, plan, scratch, idx->dev_err, &lists, st);
+  if (e != cudaSuccess) return cuda_fail(e, "search kernel");
+  e = launch_merge(lists, q, k, out_ids, out_scores, st);
+  if (e != cudaSuccess) return cuda_fail(e, "merge kernel");
+  idx->last_path = path;
+  return end_call(idx, st);
+}
