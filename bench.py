@@ -45,12 +45,14 @@ KERNEL_SOURCES = ["common.cuh", "search_tc.cuh", "search_simt.cuh", "merge.cu", 
 def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=20)
-    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--config", type=int, default=1)
     p.add_argument("--batch", type=int, default=None)
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--block-n", type=int, default=0, help="tensor-core tile rows (0 = auto)")
+    p.add_argument("--path", choices=["auto", "simt", "tc"], default="auto")
     return p.parse_args()
 
 
@@ -271,6 +273,8 @@ def run_ours(args, rank: int, world: int, local_rank: int):
         idx.set_sparse(w.doc_indptr, w.doc_terms, w.vocab, w.k1, w.b)
         q_indptr = torch.from_numpy(w.q_indptr).to(dev)
         q_terms = torch.from_numpy(w.q_terms).to(dev)
+    idx.force_block_n(args.block_n or None)
+    idx.force_path(None if args.path == "auto" else args.path)
     idx.reserve(w.q, w.k)
     idx.enable_timing(True)
     Q = to_dev(w.Q_data)

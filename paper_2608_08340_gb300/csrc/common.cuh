@@ -210,7 +210,8 @@ struct BufTopK {
       const uint64_t kth = __shfl_sync(0xffffffffu, v[(K - 1) % kE], (K - 1) / kE);
       if (lane == src) {
         count = c < K ? c : K;
-        worst = c >= K ? kth : kEmptyKey;
+        // Every kept key beats the old floor, so the floor only rises.
+        if (c >= K) worst = kth;
         floor = key_floor(worst);
       }
       __syncwarp();

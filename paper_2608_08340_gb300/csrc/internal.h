@@ -29,6 +29,7 @@ struct ListSet {
   int C = 0;
   int qt = 0;
   int sets = 1;
+  int klen = 1 << 30;   // sorted keys held per list (the merge reads min(k, klen))
 };
 
 // Optional lexical part of the fused score (Sec. 4.4 weighted fusion):
@@ -63,18 +64,24 @@ struct TcPlan {
   int nt;          // corpus tiles
   int win;         // corpus tiles per L2 window
   int pmax;        // lists per query tile
+  int tile_stride; // corpus tiles skipped between scanned tiles (1 = all)
   int stages;
   size_t smem;
 };
-TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n);
+// tile_stride > 1 scans only corpus tiles t = 0, stride, 2 * stride, ...
+TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_stride = 1);
 size_t tc_scratch_bytes(const SearchShape& s, const TcPlan& p);
+// init_floor (optional, q floats): a lower bound on each query's k-th best
+// score; lists start with it as their admission floor.
 cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s, const Fusion& fu,
                              const TcPlan& plan, void* scratch, int* dev_err, ListSet* lists,
-                             cudaStream_t st);
+                             cudaStream_t st, const float* init_floor = nullptr);
 
 // --- final merge of partial lists into the sorted top-k per query.
+// kth_out (optional, q floats): the k-th best merged score of every query
+// (-inf when fewer than k candidates exist).
 cudaError_t launch_merge(const ListSet& ls, int q, int k, int64_t* out_ids, float* out_scores,
-                         cudaStream_t st);
+                         cudaStream_t st, float* kth_out = nullptr);
 
 // --- BM25 matrix pass (lexical part of the hybrid search).
 struct SparseIndex {

@@ -33,9 +33,12 @@ __device__ __forceinline__ void offer32(WarpMerger<KP>& m, uint64_t key) {
 template <int KP>
 __global__ void __launch_bounds__(kMergeWarps * 32)
 merge_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
-             float* __restrict__ out_scores) {
+             float* __restrict__ out_scores, float* __restrict__ kth_out) {
   constexpr int kCap = 2 * KP;
   extern __shared__ __align__(16) uint64_t smem_keys[];
+  // Launched as a programmatic dependent of the search kernel: wait until
+  // that grid has finished and its lists are visible.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int qi = blockIdx.x;
   if (qi >= q) return;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -48,7 +51,8 @@ merge_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
     c0 = c0 < 0 ? 0 : c0;
     np = min(ls.P, (ls.C - c0) * ls.sets);
   }
-  const int total = np * k;
+  const int kl = min(k, ls.klen);         // keys read from each list
+  const int total = np * kl;
   const int lo = static_cast<int>(static_cast<int64_t>(total) * warp / kMergeWarps);
   const int hi = static_cast<int>(static_cast<int64_t>(total) * (warp + 1) / kMergeWarps);
 
@@ -61,8 +65,8 @@ merge_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
       const int i = g + u * 32 + lane;
       key[u] = kEmptyKey;
       if (i < hi) {
-        const int p = i / k;
-        key[u] = base[p * list_step + (i - p * k)];
+        const int p = i / kl;
+        key[u] = base[p * list_step + (i - p * kl)];
       }
     }
 #pragma unroll
@@ -90,6 +94,10 @@ merge_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
     for (int u = 0; u < kUnroll; ++u) offer32(f, key[u]);
   }
   f.finish();
+  if (kth_out != nullptr && lane == 0) {
+    const uint64_t kk = f.sbuf[k - 1];
+    kth_out[qi] = kk == kEmptyKey ? -INFINITY : key_score(kk);
+  }
   for (int i = lane; i < k; i += 32) {
     const uint64_t key = f.sbuf[i];
     const int64_t o = static_cast<int64_t>(qi) * k + i;
@@ -100,21 +108,30 @@ merge_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
 
 template <int KP>
 cudaError_t launch_merge_kp(const ListSet& ls, int q, int k, int64_t* ids, float* scores,
-                            cudaStream_t st) {
+                            cudaStream_t st, float* kth_out) {
   const size_t smem = static_cast<size_t>(kMergeWarps + 1) * 2 * KP * sizeof(uint64_t);
-  merge_kernel<KP><<<q, kMergeWarps * 32, smem, st>>>(ls, q, k, ids, scores);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(q);
+  cfg.blockDim = dim3(kMergeWarps * 32);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, merge_kernel<KP>, ls, q, k, ids, scores, kth_out);
 }
 
 }  // namespace
 
 cudaError_t launch_merge(const ListSet& ls, int q, int k, int64_t* out_ids, float* out_scores,
-                         cudaStream_t st) {
+                         cudaStream_t st, float* kth_out) {
   if (q <= 0) return cudaSuccess;
-  if (k <= 32) return launch_merge_kp<32>(ls, q, k, out_ids, out_scores, st);
-  if (k <= 64) return launch_merge_kp<64>(ls, q, k, out_ids, out_scores, st);
-  if (k <= 128) return launch_merge_kp<128>(ls, q, k, out_ids, out_scores, st);
-  return launch_merge_kp<256>(ls, q, k, out_ids, out_scores, st);
+  if (k <= 32) return launch_merge_kp<32>(ls, q, k, out_ids, out_scores, st, kth_out);
+  if (k <= 64) return launch_merge_kp<64>(ls, q, k, out_ids, out_scores, st, kth_out);
+  if (k <= 128) return launch_merge_kp<128>(ls, q, k, out_ids, out_scores, st, kth_out);
+  return launch_merge_kp<256>(ls, q, k, out_ids, out_scores, st, kth_out);
 }
 
 }  // namespace oprag

@@ -54,8 +54,9 @@ struct DeviceGuard {
   }
 };
 
-// bf16 queries with at most this many rows take the SIMT stream by default.
-constexpr int kSimtMaxQueriesBf16 = 4;
+// bf16 searches always take the tensor-core kernel (measured faster than the
+// SIMT stream even for a single query); fp32 indices take the SIMT kernel.
+constexpr int kSimtMaxQueriesBf16 = 0;
 // Largest BM25 matrix block (floats) materialised per hybrid pass.
 constexpr int64_t kLexMaxElems = int64_t(1) << 28;
 
@@ -168,11 +169,43 @@ int run_search(oprag_index* idx, const void* Q, int q, int k, const Fusion& fu, 
     e = launch_simt_search(idx->dtype, idx->emb, Q, s, fu, idx->scratch, grid, &lists, st);
   } else {
     const TcPlan plan = tc_plan(s, idx->num_sms, idx->opt_block_n);
-    int rc = idx->ensure(&idx->scratch, &idx->scratch_bytes, tc_scratch_bytes(s, plan),
+    const size_t main_bytes = (tc_scratch_bytes(s, plan) + 255) / 256 * 256;
+    // Buffered lists (k > 32) collect every score above their floor, and the
+    // floor of a fresh list starts at -inf.  A cheap first pass over every
+    // kSampleStride-th corpus tile with 32-key lists yields, per query, the
+    // k-th best of real corpus scores -- a lower bound of the true k-th best
+    // -- which the main pass then uses as the lists' starting floor.
+    constexpr int kSampleStride = 16;
+    const bool sampled = list_len_for(k) > 32 && plan.nt >= 8 * kSampleStride;
+    SearchShape s32 = s;
+    s32.k = 32;
+    TcPlan splan{};
+    size_t sample_bytes = 0;
+    if (sampled) {
+      splan = tc_plan(s32, idx->num_sms, plan.block_n, kSampleStride);
+      sample_bytes = (tc_scratch_bytes(s32, splan) + 255) / 256 * 256 +
+                     (static_cast<size_t>(q) * k * 12 + 255) / 256 * 256 +
+                     static_cast<size_t>(q) * sizeof(float);
+    }
+    int rc = idx->ensure(&idx->scratch, &idx->scratch_bytes, main_bytes + sample_bytes,
                          "search scratch");
     if (rc) return rc;
     if (idx->timing) cudaEventRecord(idx->ev[1], st);
-    e = launch_tc_search(idx->emb, Q, s, fu, plan, idx->scratch, idx->dev_err, &lists, st);
+    const float* floor = nullptr;
+    if (sampled) {
+      char* sbase = static_cast<char*>(idx->scratch) + main_bytes;
+      const size_t slist = (tc_scratch_bytes(s32, splan) + 255) / 256 * 256;
+      int64_t* sids = reinterpret_cast<int64_t*>(sbase + slist);
+      float* sscores = reinterpret_cast<float*>(sids + static_cast<size_t>(q) * k);
+      float* kth = reinterpret_cast<float*>(
+          sbase + slist + (static_cast<size_t>(q) * k * 12 + 255) / 256 * 256);
+      ListSet slists{};
+      e = launch_tc_search(idx->emb, Q, s32, fu, splan, sbase, idx->dev_err, &slists, st);
+      if (e == cudaSuccess) e = launch_merge(slists, q, k, sids, sscores, st, kth);
+      if (e != cudaSuccess) return cuda_fail(e, "sampling pass");
+      floor = kth;
+    }
+    e = launch_tc_search(idx->emb, Q, s, fu, plan, idx->scratch, idx->dev_err, &lists, st, floor);
   }
   if (e != cudaSuccess) return cuda_fail(e, "search kernel");
   if (idx->timing) cudaEventRecord(idx->ev[2], st);

@@ -113,6 +113,7 @@ simt_search_kernel(const T* __restrict__ E, int64_t n, int d, const T* __restric
   const int q0 = chunk * QC;
   const int nq = min(QC, q - q0);
 
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   for (int i = threadIdx.x; i < QC * d; i += blockDim.x) {
     const int qq = i / d, j = i % d;
     qs[i] = qq < nq ? to_f32<T>(Q[static_cast<int64_t>(q0 + qq) * d + j]) : 0.f;
@@ -247,6 +248,7 @@ cudaError_t launch_t(const void* E, const void* Q, const SearchShape& s, const F
   lists->P = grid;
   lists->TH = QC;
   lists->stride = K;
+  lists->klen = K;
   return cudaGetLastError();
 }
 

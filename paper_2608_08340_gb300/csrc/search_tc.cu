@@ -49,7 +49,7 @@ bool make_map(CUtensorMap* m, const void* base, int64_t rows, int d, int box_row
 
 }  // namespace
 
-TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n) {
+TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_stride) {
   TcPlan pl{};
   pl.qt = (s.q + kBlockM - 1) / kBlockM;
   int bn = 256;
@@ -62,7 +62,9 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n) {
     if (units256 < 4LL * num_sms) bn = 128;
   }
   pl.block_n = bn;
-  pl.nt = static_cast<int>((s.n + bn - 1) / bn);
+  pl.tile_stride = tile_stride < 1 ? 1 : tile_stride;
+  const int64_t all_tiles = (s.n + bn - 1) / bn;
+  pl.nt = static_cast<int>((all_tiles + pl.tile_stride - 1) / pl.tile_stride);
   const int64_t units = static_cast<int64_t>(pl.nt) * pl.qt;
   pl.grid = static_cast<int>(units < num_sms ? units : num_sms);
   if (pl.grid < 1) pl.grid = 1;
@@ -111,9 +113,13 @@ size_t tc_scratch_bytes(const SearchShape& s, const TcPlan& pl) {
 
 cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s, const Fusion& fu,
                              const TcPlan& pl, void* scratch, int* dev_err, ListSet* lists,
-                             cudaStream_t st) {
+                             cudaStream_t st, const float* init_floor) {
   CUtensorMap mq, me;
-  if (!make_map(&mq, Q, s.q, s.d, kBlockM) || !make_map(&me, E, s.n, s.d, pl.block_n))
+  // With a single query tile only its real rows are loaded (the remaining
+  // rows of the A tile hold stale data whose TMEM lanes the epilogue never
+  // reads); rows are loaded in multiples of 8, the swizzle atom height.
+  const int a_rows = pl.qt == 1 ? std::min(kBlockM, (s.q + 7) / 8 * 8) : kBlockM;
+  if (!make_map(&mq, Q, s.q, s.d, a_rows) || !make_map(&me, E, s.n, s.d, pl.block_n))
     return cudaErrorInvalidValue;
   const int K = list_len_for(s.k);
   const int stride = K > 32 ? 2 * K : K;
@@ -128,6 +134,9 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
   prm.win = pl.win;
   prm.pmax = pl.pmax;
   prm.kblocks = (s.d + kBlockK - 1) / kBlockK;
+  prm.a_bytes = static_cast<uint32_t>(a_rows) * kBlockK * 2;
+  prm.tile_stride = pl.tile_stride;
+  prm.init_floor = init_floor;
   prm.fu = fu;
   prm.lists = static_cast<uint64_t*>(scratch);
   prm.meta_worst = prm.lists + rows * stride;
@@ -140,6 +149,7 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
   lists->C = pl.grid;
   lists->qt = pl.qt;
   lists->sets = epi_sets(K);
+  lists->klen = K;
   const bool hybrid = fu.bm25 != nullptr;
   if (pl.block_n == 128) return launch_bn128(mq, me, prm, pl.grid, hybrid, st);
   return hybrid ? launch_bn256_fused(mq, me, prm, pl.grid, st)

@@ -56,6 +56,9 @@ struct TcParams {
   int win;              // corpus tiles per L2 window
   int pmax;             // lists per query tile (CTAs that may touch it x kEpiSets)
   int kblocks;
+  uint32_t a_bytes;     // bytes of one query K block actually loaded (rows x 128)
+  int tile_stride;      // scanned corpus tile i is tile i * tile_stride
+  const float* init_floor;  // optional per-query lower bound of the k-th best score
   Fusion fu;
   uint64_t* lists;      // [(j * pmax + producer) * 128 + row] * stride
   int* meta_count;      // buffered lists: kept keys per (list, row)
@@ -79,6 +82,7 @@ struct UnitSeq {
     nt = p.nt;
     win = p.win;
     qt = p.qt;
+    stride = p.tile_stride;
     C = C_;
     cta = cta_;
     w = -1;
@@ -103,7 +107,8 @@ struct UnitSeq {
     if (++l >= l_end) next_window();
   }
   __device__ __forceinline__ int j() const { return static_cast<int>(l / tw); }
-  __device__ __forceinline__ int t() const { return w * win + static_cast<int>(l % tw); }
+  __device__ __forceinline__ int t() const { return (w * win + static_cast<int>(l % tw)) * stride; }
+  int stride;
 };
 
 // First CTA whose shares can reach query tile j (the host checks the bound).
@@ -261,7 +266,7 @@ template <int K>
 struct EpiList<K, false> {
   static constexpr int kStride = K;
   RegTopK<K> t;
-  __device__ __forceinline__ void init_mem(const TcParams& p, int64_t sr) {
+  __device__ __forceinline__ void init_mem(const TcParams& p, int64_t sr, int) {
 #pragma unroll
     for (int i = 0; i < K; i += 2)
       *reinterpret_cast<ulonglong2*>(p.lists + sr * K + i) = make_ulonglong2(0ull, 0ull);
@@ -281,9 +286,12 @@ template <int K>
 struct EpiList<K, true> {
   static constexpr int kStride = 2 * K;
   BufTopK<K> t;
-  __device__ __forceinline__ void init_mem(const TcParams& p, int64_t sr) {
+  __device__ __forceinline__ void init_mem(const TcParams& p, int64_t sr, int qidx) {
     p.meta_count[sr] = 0;
-    p.meta_worst[sr] = kEmptyKey;
+    // A known lower bound f of the k-th best score admits only scores >= f
+    // (the key with the largest possible id ranks below every such score).
+    const float f = p.init_floor != nullptr ? p.init_floor[qidx] : -INFINITY;
+    p.meta_worst[sr] = f > -INFINITY ? make_key(f, kNoId) : kEmptyKey;
   }
   __device__ __forceinline__ void load(const TcParams& p, int64_t sr) {
     t.buf = p.lists + sr * kStride;
@@ -357,11 +365,30 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     prefetch_map(&map_q);
     prefetch_map(&map_e);
   }
+  int pre_issued = 0;           // stages the producer issued before the setup barrier
+  if (threadIdx.x == 0) {
+    // The ring is empty: start the first loads while TMEM is being allocated.
+    UnitSeq us;
+    us.start(p, cta, C);
+    for (; us.valid() && pre_issued < S; us.next()) {
+      for (int kb = 0; kb < p.kblocks && pre_issued < S; ++kb, ++pre_issued) {
+        mbar_arrive_expect_tx(&full[pre_issued], p.a_bytes + kBStageBytes);
+        tma_load_2d(sA + pre_issued * kAStageBytes, &map_q, &full[pre_issued], kb * kBlockK,
+                    us.j() * kBlockM);
+        tma_load_2d(sB + pre_issued * kBStageBytes, &map_e, &full[pre_issued], kb * kBlockK,
+                    us.t() * BN);
+      }
+      if (pre_issued >= S) break;
+    }
+  }
   if (warp == 1) tmem_alloc(tmem_slot, kTmemCols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  // Let the merge kernel that follows on the stream get scheduled; it waits
+  // for this grid to finish before reading the lists.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (warp == 0) {
     if (lane == 0) {
@@ -370,13 +397,21 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       uint32_t ph = 0;
       uint32_t issued = 0, parity = 0;    // per stage: ever issued, parity of last issue
       bool ok = true;
+      int skip = pre_issued;              // already issued before the setup barrier
       UnitSeq us;
       for (us.start(p, cta, C); ok && us.valid(); us.next()) {
         const int j = us.j();
         const int t = us.t();
         for (int kb = 0; kb < p.kblocks; ++kb) {
+          if (skip > 0) {
+            --skip;
+            issued |= 1u << s;
+            parity &= ~(1u << s);
+            if (++s == S) { s = 0; ph ^= 1u; }
+            continue;
+          }
           if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, p.dev_err)) { ok = false; break; }
-          mbar_arrive_expect_tx(&full[s], kAStageBytes + kBStageBytes);
+          mbar_arrive_expect_tx(&full[s], p.a_bytes + kBStageBytes);
           tma_load_2d(sA + s * kAStageBytes, &map_q, &full[s], kb * kBlockK, j * kBlockM);
           tma_load_2d(sB + s * kBStageBytes, &map_e, &full[s], kb * kBlockK, t * BN);
           issued |= 1u << s;
@@ -443,7 +478,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
 
     // This CTA owns the list slots (j, cta - first_cta(j)); empty them first.
     for (int j = 0; j < p.qt; ++j)
-      if (owns(j) && j * kBlockM + row < p.q) list.init_mem(p, list_row(j));
+      if (owns(j) && j * kBlockM + row < p.q) list.init_mem(p, list_row(j), j * kBlockM + row);
 
     int cur_j = -1;
     int64_t cur_sr = 0;

@@ -199,3 +199,20 @@ def test_config4_scale_with_upserts_sampled():
     got = idx.rows().view(torch.int16).numpy().view(np.uint16)
     np.testing.assert_array_equal(got, E)
     idx.check()
+
+
+@pytest.mark.parametrize("k", [33, 100, 256])
+def test_large_k_with_sampled_floor(k):
+    """k > 32 over many corpus tiles: the search first scans every 16th tile
+    to get a lower bound of each query's k-th best score, then the full scan
+    admits only scores above it.  Results must still be exact."""
+    rng = np.random.default_rng(k)
+    n, d, q = 160000, 128, 130
+    E = workloads.to_bf16_bits(workloads._normalise(rng.standard_normal((n, d)).astype(np.float32)))
+    Q = workloads.to_bf16_bits(workloads._normalise(rng.standard_normal((q, d)).astype(np.float32)))
+    idx = _index(E)
+    ids, sc = idx.search(dev_tensor(Q), k)
+    assert idx.last_path == "tc"
+    rows = np.sort(rng.choice(q, 12, replace=False))
+    check_dense(ids, sc, E, Q, k, f"large k={k}", rows=rows)
+    idx.check()
