@@ -4,7 +4,8 @@
 // Op_retrieve (Sec. 3.2; Sec. 4.1 Retrieval), done inside one GPU: the
 // producers are corpus slices instead of index shards.
 //
-// One CTA per query.  The P * k candidate keys of a query (the first k of each
+// Many lists (more than 32 per query): one CTA per query.  The P * k
+// candidate keys of a query (the first k of each
 // producer's sorted list) are split evenly over the warps; a warp fetches four
 // 32-key groups at once (independent loads, so L2 latency is paid once per
 // group of four, not once per list) and filters them against its running
@@ -123,11 +124,90 @@ cudaError_t launch_merge_kp(const ListSet& ls, int q, int k, int64_t* ids, float
   return cudaLaunchKernelEx(&cfg, merge_kernel<KP>, ls, q, k, ids, scores, kth_out);
 }
 
+// Few lists per query (at most 32): one warp per query merges the sorted
+// lists directly.  Lane l holds the head of list l (with the next keys
+// prefetched in registers); each round the warp takes the largest head
+// (keys are unique, so exactly one lane wins) and that lane advances.
+constexpr int kHeads = 16;          // keys prefetched per list
+constexpr int kWayWarps = 8;        // queries per CTA
+
+__global__ void __launch_bounds__(kWayWarps * 32)
+merge_kway_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
+                  float* __restrict__ out_scores, float* __restrict__ kth_out) {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qi = blockIdx.x * kWayWarps + warp;
+  if (qi >= q) return;
+  const int tile = qi / ls.TH, row = qi % ls.TH;
+  int np = ls.P;
+  if (ls.C > 0) {
+    int c0 = static_cast<int>(static_cast<int64_t>(tile) * ls.C / ls.qt) - 1;
+    c0 = c0 < 0 ? 0 : c0;
+    np = min(ls.P, (ls.C - c0) * ls.sets);
+  }
+  const int kl = min(k, ls.klen);
+  const uint64_t* list = ls.keys + ((static_cast<int64_t>(tile) * ls.P + lane) * ls.TH + row) *
+                                       static_cast<int64_t>(ls.stride);
+  const bool has_list = lane < np;
+  uint64_t h[kHeads];
+  int next = 0;       // keys of this list fetched so far
+  auto refill = [&]() {
+#pragma unroll
+    for (int i = 0; i < kHeads; ++i) h[i] = next + i < kl ? list[next + i] : kEmptyKey;
+    next += kHeads;
+  };
+  if (has_list) refill();
+  else {
+#pragma unroll
+    for (int i = 0; i < kHeads; ++i) h[i] = kEmptyKey;
+  }
+  int avail = kHeads;
+  uint64_t mine = kEmptyKey;      // the answer of rank (lane + 32 * m) for the current m
+  for (int r = 0; r < k; ++r) {
+    uint64_t best = h[0];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) best = umax64(best, __shfl_xor_sync(0xffffffffu, best, o));
+    if (best != kEmptyKey && h[0] == best) {
+#pragma unroll
+      for (int i = 0; i + 1 < kHeads; ++i) h[i] = h[i + 1];
+      h[kHeads - 1] = kEmptyKey;
+      if (--avail == 0 && next < kl) {
+        refill();
+        avail = kHeads;
+      }
+    }
+    if ((r & 31) == lane) mine = best;
+    if ((r & 31) == 31 || r == k - 1) {
+      const int i = (r & ~31) + lane;
+      if (i <= r) {
+        const int64_t o = static_cast<int64_t>(qi) * k + i;
+        out_ids[o] = mine == kEmptyKey ? -1 : static_cast<int64_t>(key_id(mine));
+        out_scores[o] = mine == kEmptyKey ? -INFINITY : key_score(mine);
+      }
+    }
+    if (r == k - 1 && kth_out != nullptr && lane == 0)
+      kth_out[qi] = best == kEmptyKey ? -INFINITY : key_score(best);
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_merge(const ListSet& ls, int q, int k, int64_t* out_ids, float* out_scores,
                          cudaStream_t st, float* kth_out) {
   if (q <= 0) return cudaSuccess;
+  if (ls.P <= 32) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3((q + kWayWarps - 1) / kWayWarps);
+    cfg.blockDim = dim3(kWayWarps * 32);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, merge_kway_kernel, ls, q, k, out_ids, out_scores, kth_out);
+  }
   if (k <= 32) return launch_merge_kp<32>(ls, q, k, out_ids, out_scores, st, kth_out);
   if (k <= 64) return launch_merge_kp<64>(ls, q, k, out_ids, out_scores, st, kth_out);
   if (k <= 128) return launch_merge_kp<128>(ls, q, k, out_ids, out_scores, st, kth_out);
