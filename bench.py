@@ -53,6 +53,8 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--block-n", type=int, default=0, help="tensor-core tile rows (0 = auto)")
     p.add_argument("--path", choices=["auto", "simt", "tc"], default="auto")
+    p.add_argument("--pair", choices=["auto", "single", "pair"], default="auto",
+                   help="tensor-core kernel: CTA pairs (M = 256 MMAs) or single CTAs")
     return p.parse_args()
 
 
@@ -275,6 +277,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
         q_terms = torch.from_numpy(w.q_terms).to(dev)
     idx.force_block_n(args.block_n or None)
     idx.force_path(None if args.path == "auto" else args.path)
+    idx.force_pair(None if args.pair == "auto" else args.pair)
     idx.reserve(w.q, w.k)
     idx.enable_timing(True)
     Q = to_dev(w.Q_data)
@@ -304,7 +307,9 @@ def run_ours(args, rank: int, world: int, local_rank: int):
         else:
             idx.search(Q, w.k, out=(ids, scores))
 
-    launches_per_step = 2 + (1 if cfg in (3, 4) else 0)
+    # search + merge; k > 32 adds the sampled first pass (search + merge);
+    # config 3 adds the BM25 pass, config 4 the upsert scatter.
+    launches_per_step = 2 + (2 if w.k > 32 else 0) + (1 if cfg in (3, 4) else 0)
 
     for i in range(args.warmup):
         flush.zero_()
@@ -417,6 +422,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
         "gpu_launches": launches_per_step * args.steps,
         "clocks": dict(clocks.summary(), smi=smi.summary()),
         "path": idx.last_path,
+        "launch": idx.last_launch,
     }
     idx.close()
     return result, w

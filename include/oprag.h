@@ -177,6 +177,12 @@ OPRAG_API int oprag_index_check(oprag_index *idx);
 #define OPRAG_OPT_BLOCK_N 2
 OPRAG_API int oprag_index_set_option(oprag_index *idx, int32_t option, int32_t value);
 
+/* OPRAG_OPT_PAIR (tensor-core path): 2 runs clusters of two CTAs that issue
+ * M = 256 MMAs together, each CTA loading half of every corpus tile (needs
+ * 256-row corpus tiles; ignored with 128-row tiles).  0 (default) and 1 run
+ * every CTA on its own (M = 128 MMAs). */
+#define OPRAG_OPT_PAIR 4
+
 /* OPRAG_OPT_TIMING: 1 makes every later search record CUDA events, on the
  * call's stream, around its lexical (BM25) kernel, its main search kernel and
  * its merge kernel; oprag_index_last_timing() reads them.  0 (default) off. */
@@ -195,6 +201,13 @@ OPRAG_API int oprag_index_last_timing(oprag_index *idx, float *lexical_ms, float
 /* Which kernel family served the last search on this index: 1 SIMT, 2 tensor
  * core, 0 none yet. */
 OPRAG_API int oprag_index_last_path(const oprag_index *idx);
+
+/* Launch shape of the last search's main tensor-core kernel: grid (CTAs),
+ * cluster (1 single CTAs, 2 CTA pairs issuing M = 256 MMAs) and block_n
+ * (corpus rows per tile); all 0 when the last search ran the SIMT kernel.
+ * Out-pointers may be NULL.  OPRAG_ERR_NOT_READY before the first search. */
+OPRAG_API int oprag_index_last_launch(const oprag_index *idx, int32_t *grid, int32_t *cluster,
+                                      int32_t *block_n);
 
 /*
  * oprag_search without any device allocation.  The paper has no counterpart:

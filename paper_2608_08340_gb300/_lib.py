@@ -15,6 +15,7 @@ OPRAG_K_MAX = 256
 OPRAG_OPT_PATH = 1
 OPRAG_OPT_BLOCK_N = 2
 OPRAG_OPT_TIMING = 3
+OPRAG_OPT_PAIR = 4
 
 ERRORS = {
     0: "OK",
@@ -48,6 +49,8 @@ SIGNATURES = {
     "oprag_index_check": (_I32, [_P]),
     "oprag_index_set_option": (_I32, [_P, _I32, _I32]),
     "oprag_index_last_path": (_I32, [_P]),
+    "oprag_index_last_launch": (_I32, [_P, ctypes.POINTER(_I32), ctypes.POINTER(_I32),
+                                       ctypes.POINTER(_I32)]),
     "oprag_index_last_timing": (_I32, [_P, ctypes.POINTER(_F), ctypes.POINTER(_F),
                                        ctypes.POINTER(_F)]),
     "oprag_last_error": (ctypes.c_char_p, []),

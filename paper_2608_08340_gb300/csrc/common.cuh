@@ -87,6 +87,23 @@ __device__ __forceinline__ void warp_sort_desc(uint64_t (&v)[E]) {
 }
 
 // ---------------------------------------------------------------------------
+// a[idx] (0 <= idx < N, N a power of two) for a register array, as a tree of
+// selects on the bits of idx, so that the array stays in registers.
+template <int N>
+__device__ __forceinline__ float reg_select(const float (&a)[N], int idx) {
+  static_assert((N & (N - 1)) == 0, "power of two");
+  float t[N];
+#pragma unroll
+  for (int i = 0; i < N; ++i) t[i] = a[i];
+#pragma unroll
+  for (int w = N / 2; w >= 1; w /= 2) {
+    const bool hi = (idx & w) != 0;
+#pragma unroll
+    for (int i = 0; i < w; ++i) t[i] = hi ? t[i + w] : t[i];
+  }
+  return t[0];
+}
+
 // Running top-K of one lane, K <= 32, kept sorted (best first) in registers as
 // (score, id) pairs.  Candidates must reach a list in increasing id order (the
 // corpus is scanned in id order), so a candidate whose score equals a kept one
@@ -111,6 +128,9 @@ struct RegTopK {
   }
 
   __device__ __forceinline__ bool full() const { return id[K - 1] != kNoId; }
+
+  // k-th best score held (1 <= k <= K); -inf while fewer than k are held.
+  __device__ __forceinline__ float kth(int k) const { return reg_select(s, k - 1); }
 
   __device__ __forceinline__ void push(float v, uint32_t vid) {
     if (v > s[K - 1]) insert(v, vid);
@@ -317,26 +337,40 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
 }
 
+// kCluster: acquire at cluster scope (the phase was completed by arrivals
+// from the other CTA of a cluster).
+template <bool kCluster = false>
 __device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(smem_addr(bar)), "r"(parity)
-      : "memory");
+  if constexpr (kCluster) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_addr(bar)), "r"(parity)
+        : "memory");
+  } else {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_addr(bar)), "r"(parity)
+        : "memory");
+  }
   return ok != 0;
 }
 
 // Waits for the phase with the given parity to complete.  Gives up when the
 // CTA-wide abort word is set or the cycle limit passes (then sets both).
+template <bool kCluster = false>
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
                                           int* dev_err) {
-  if (mbar_test(bar, parity)) return true;
+  if (mbar_test<kCluster>(bar, parity)) return true;
   const long long t0 = clock64();
   while (true) {
-    if (mbar_test(bar, parity)) return true;
+    if (mbar_test<kCluster>(bar, parity)) return true;
     if (*abort_flag) return false;
     if (clock64() - t0 > kWaitLimitCycles) {
       *abort_flag = 1;

@@ -24,11 +24,14 @@ struct ListSet {
   int P;
   int TH;
   int stride;
-  // Tensor-core lists: only producers p < sets * (C - first_cta(tile)) exist
-  // for a tile (see search_tc.cuh); C == 0 means all P lists exist.
+  // Tensor-core lists: only producers p < sets * (C - first_cta(tile / pair))
+  // exist for a tile (see search_tc.cuh); C == 0 means all P lists exist.
+  // C and qt count the kernel's schedule units: CTAs (pairs of CTAs) and
+  // query tiles (pairs of query tiles) when pair == 1 (2).
   int C = 0;
   int qt = 0;
   int sets = 1;
+  int pair = 1;
   int klen = 1 << 30;   // sorted keys held per list (the merge reads min(k, klen))
 };
 
@@ -60,7 +63,9 @@ cudaError_t launch_simt_search(int dtype, const void* E, const void* Q, const Se
 struct TcPlan {
   int block_n;     // corpus rows per tile: 128 or 256
   int grid;        // CTAs (persistent)
+  int pair;        // 2: clusters of two CTAs issue M = 256 MMAs together; 1: single CTAs
   int qt;          // query tiles of 128
+  int uqt;         // query tiles of the schedule: qt, or ceil(qt / 2) pairs of tiles
   int nt;          // corpus tiles
   int win;         // corpus tiles per L2 window
   int pmax;        // lists per query tile
@@ -69,13 +74,22 @@ struct TcPlan {
   size_t smem;
 };
 // tile_stride > 1 scans only corpus tiles t = 0, stride, 2 * stride, ...
-TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_stride = 1);
+// force_pair: 0 automatic, 1 single CTAs, 2 CTA pairs (needs 256-row tiles).
+// pair_capacity: clusters of two that fit on the device (0: no pair mode).
+TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_stride = 1,
+               int force_pair = 0, int pair_capacity = 0);
+// Clusters of two pair-mode CTAs that fit on the current device at once.
+int tc_pair_capacity();
 size_t tc_scratch_bytes(const SearchShape& s, const TcPlan& p);
 // init_floor (optional, q floats): a lower bound on each query's k-th best
 // score; lists start with it as their admission floor.
+// qfloor (optional, q entries, register lists only): per-query k-th score
+// bounds shared by all lists, valid for entries tagged with gen (see
+// search_tc.cuh); zero-filled memory is a valid initial state.
 cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s, const Fusion& fu,
                              const TcPlan& plan, void* scratch, int* dev_err, ListSet* lists,
-                             cudaStream_t st, const float* init_floor = nullptr);
+                             cudaStream_t st, const float* init_floor = nullptr,
+                             uint64_t* qfloor = nullptr, uint32_t gen = 0);
 
 // --- final merge of partial lists into the sorted top-k per query.
 // kth_out (optional, q floats): the k-th best merged score of every query

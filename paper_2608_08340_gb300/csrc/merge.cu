@@ -48,7 +48,7 @@ merge_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
   const int64_t list_step = static_cast<int64_t>(ls.TH) * ls.stride;
   int np = ls.P;
   if (ls.C > 0) {
-    int c0 = static_cast<int>(static_cast<int64_t>(tile) * ls.C / ls.qt) - 1;
+    int c0 = static_cast<int>(static_cast<int64_t>(tile / ls.pair) * ls.C / ls.qt) - 1;
     c0 = c0 < 0 ? 0 : c0;
     np = min(ls.P, (ls.C - c0) * ls.sets);
   }
@@ -141,7 +141,7 @@ merge_kway_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
   const int tile = qi / ls.TH, row = qi % ls.TH;
   int np = ls.P;
   if (ls.C > 0) {
-    int c0 = static_cast<int>(static_cast<int64_t>(tile) * ls.C / ls.qt) - 1;
+    int c0 = static_cast<int>(static_cast<int64_t>(tile / ls.pair) * ls.C / ls.qt) - 1;
     c0 = c0 < 0 ? 0 : c0;
     np = min(ls.P, (ls.C - c0) * ls.sets);
   }

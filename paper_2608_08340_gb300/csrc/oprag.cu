@@ -88,7 +88,15 @@ struct oprag_index {
 
   int opt_path = 0;
   int opt_block_n = 0;
+  int opt_pair = 0;
+  // Per-query k-th score bounds shared by the lists of one search, tagged
+  // with a per-launch generation (zeroed memory holds no valid entry).
+  uint64_t* qfloor = nullptr;
+  size_t qfloor_bytes = 0;
+  uint32_t gen = 0;
+  int pair_cap = -1;       // clusters of two search CTAs that fit at once (-1: not asked yet)
   int last_path = 0;
+  int last_grid = 0, last_cluster = 0, last_block_n = 0;   // last main search kernel launch
 
   // Optional kernel timing: events before the lexical pass, before the
   // search kernel, before the merge kernel and after it.
@@ -147,6 +155,48 @@ int end_call(oprag_index* idx, cudaStream_t st) {
   return ok();
 }
 
+// Clusters of two pair-mode search CTAs that fit at once on the index's
+// device; asked once (the device is current inside every entry point).
+int pair_capacity(oprag_index* idx) {
+  if (idx->pair_cap < 0) {
+    idx->pair_cap = tc_pair_capacity();
+    cudaGetLastError();
+  }
+  return idx->pair_cap;
+}
+
+// Shared k-th score bounds for a search of q queries: grows (and zeroes) the
+// per-index array and hands out a fresh generation tag.
+int shared_floors(oprag_index* idx, int q, cudaStream_t st, uint64_t** qf, uint32_t* gen) {
+  const size_t need = static_cast<size_t>(q) * sizeof(uint64_t);
+  if (need > idx->qfloor_bytes) {
+    int rc = idx->ensure(reinterpret_cast<void**>(&idx->qfloor), &idx->qfloor_bytes, need,
+                         "shared k-th score bounds");
+    if (rc) return rc;
+    cudaError_t e = cudaMemsetAsync(idx->qfloor, 0, idx->qfloor_bytes, st);
+    if (e != cudaSuccess) return cuda_fail(e, "clearing shared bounds");
+  }
+  if (++idx->gen == 0) {            // tags wrapped: old entries could read as current
+    cudaError_t e = cudaMemsetAsync(idx->qfloor, 0, idx->qfloor_bytes, st);
+    if (e != cudaSuccess) return cuda_fail(e, "clearing shared bounds");
+    idx->gen = 1;
+  }
+  *qf = idx->qfloor;
+  *gen = idx->gen;
+  return OPRAG_OK;
+}
+
+// Records the shape of a search's main kernel launch (oprag_index_last_launch).
+void note_launch(oprag_index* idx, int path, const TcPlan& plan) {
+  if (path == 2) {
+    idx->last_grid = plan.grid;
+    idx->last_cluster = plan.pair;
+    idx->last_block_n = plan.block_n;
+  } else {
+    idx->last_grid = idx->last_cluster = idx->last_block_n = 0;
+  }
+}
+
 int choose_path(const oprag_index* idx, int q) {
   if (idx->dtype == OPRAG_F32) return 1;
   if (idx->opt_path == 1 || idx->opt_path == 2) return idx->opt_path;
@@ -159,6 +209,7 @@ int run_search(oprag_index* idx, const void* Q, int q, int k, const Fusion& fu, 
   SearchShape s{idx->n, idx->d, q, k};
   const int path = choose_path(idx, q);
   ListSet lists{};
+  TcPlan plan_used{};
   cudaError_t e;
   if (path == 1) {
     const int grid = simt_grid(s, idx->num_sms);
@@ -168,7 +219,7 @@ int run_search(oprag_index* idx, const void* Q, int q, int k, const Fusion& fu, 
     if (idx->timing) cudaEventRecord(idx->ev[1], st);
     e = launch_simt_search(idx->dtype, idx->emb, Q, s, fu, idx->scratch, grid, &lists, st);
   } else {
-    const TcPlan plan = tc_plan(s, idx->num_sms, idx->opt_block_n);
+    const TcPlan plan = tc_plan(s, idx->num_sms, idx->opt_block_n, 1, idx->opt_pair, pair_capacity(idx));
     const size_t main_bytes = (tc_scratch_bytes(s, plan) + 255) / 256 * 256;
     // Buffered lists (k > 32) collect every score above their floor, and the
     // floor of a fresh list starts at -inf.  A cheap first pass over every
@@ -182,7 +233,7 @@ int run_search(oprag_index* idx, const void* Q, int q, int k, const Fusion& fu, 
     TcPlan splan{};
     size_t sample_bytes = 0;
     if (sampled) {
-      splan = tc_plan(s32, idx->num_sms, plan.block_n, kSampleStride);
+      splan = tc_plan(s32, idx->num_sms, plan.block_n, kSampleStride, plan.pair, pair_capacity(idx));
       sample_bytes = (tc_scratch_bytes(s32, splan) + 255) / 256 * 256 +
                      (static_cast<size_t>(q) * k * 12 + 255) / 256 * 256 +
                      static_cast<size_t>(q) * sizeof(float);
@@ -205,10 +256,18 @@ int run_search(oprag_index* idx, const void* Q, int q, int k, const Fusion& fu, 
       if (e != cudaSuccess) return cuda_fail(e, "sampling pass");
       floor = kth;
     }
-    e = launch_tc_search(idx->emb, Q, s, fu, plan, idx->scratch, idx->dev_err, &lists, st, floor);
+    uint64_t* qf = nullptr;
+    uint32_t gen = 0;
+    if (list_len_for(k) <= 32) {
+      if ((rc = shared_floors(idx, q, st, &qf, &gen))) return rc;
+    }
+    e = launch_tc_search(idx->emb, Q, s, fu, plan, idx->scratch, idx->dev_err, &lists, st, floor,
+                         qf, gen);
+    plan_used = plan;
   }
   if (e != cudaSuccess) return cuda_fail(e, "search kernel");
   if (idx->timing) cudaEventRecord(idx->ev[2], st);
+  note_launch(idx, path, plan_used);
   e = launch_merge(lists, q, k, out_ids, out_scores, st);
   if (e != cudaSuccess) return cuda_fail(e, "merge kernel");
   if (idx->timing) cudaEventRecord(idx->ev[3], st);
@@ -321,6 +380,7 @@ void oprag_index_destroy(oprag_index* idx) {
   if (idx->emb) cudaFree(idx->emb);
   if (idx->dev_err) cudaFree(idx->dev_err);
   if (idx->scratch) cudaFree(idx->scratch);
+  if (idx->qfloor) cudaFree(idx->qfloor);
   if (idx->lex) cudaFree(idx->lex);
   if (idx->stage) cudaFree(idx->stage);
   idx->free_sparse();
@@ -368,7 +428,9 @@ int oprag_index_reserve(oprag_index* idx, int32_t q_max, int32_t k_max) {
       for (int qq : {q_max, std::min(q_max, 128)}) {
         SearchShape s2 = s;
         s2.q = qq;
-        need = std::max(need, tc_scratch_bytes(s2, tc_plan(s2, idx->num_sms, bn)));
+        for (int pair : {1, 2})
+          need = std::max(need, tc_scratch_bytes(s2, tc_plan(s2, idx->num_sms, bn, 1, pair,
+                                                             pair_capacity(idx))));
       }
     }
   }
@@ -640,6 +702,11 @@ int oprag_index_set_option(oprag_index* idx, int32_t option, int32_t value) {
     idx->timing = value != 0;
     return ok();
   }
+  if (option == OPRAG_OPT_PAIR) {
+    if (value < 0 || value > 2) return fail(OPRAG_ERR_INVALID_ARG, "pair mode %d", value);
+    idx->opt_pair = value;
+    return ok();
+  }
   if (option == OPRAG_OPT_BLOCK_N) {
     if (value != 0 && value != 128 && value != 256)
       return fail(OPRAG_ERR_INVALID_ARG, "block_n %d", value);
@@ -650,6 +717,16 @@ int oprag_index_set_option(oprag_index* idx, int32_t option, int32_t value) {
 }
 
 int oprag_index_last_path(const oprag_index* idx) { return idx ? idx->last_path : 0; }
+
+int oprag_index_last_launch(const oprag_index* idx, int32_t* grid, int32_t* cluster,
+                            int32_t* block_n) {
+  if (!idx) return fail(OPRAG_ERR_INVALID_ARG, "index is NULL");
+  if (!idx->last_path) return fail(OPRAG_ERR_NOT_READY, "no search was issued");
+  if (grid) *grid = idx->last_grid;
+  if (cluster) *cluster = idx->last_cluster;
+  if (block_n) *block_n = idx->last_block_n;
+  return ok();
+}
 
 int oprag_index_last_timing(oprag_index* idx, float* lexical_ms, float* search_ms,
                             float* merge_ms) {
@@ -728,7 +805,7 @@ extern "C" int oprag_search_noalloc(oprag_index* idx, const void* queries, int32
     grid = simt_grid(s, idx->num_sms);
     need = simt_scratch_bytes(idx->dtype, s, grid);
   } else {
-    plan = tc_plan(s, idx->num_sms, idx->opt_block_n);
+    plan = tc_plan(s, idx->num_sms, idx->opt_block_n, 1, idx->opt_pair, pair_capacity(idx));
     need = tc_scratch_bytes(s, plan);
   }
   if (need > kStaticScratchBytes)
@@ -743,6 +820,7 @@ extern "C" int oprag_search_noalloc(oprag_index* idx, const void* queries, int32
       path == 1 ? launch_simt_search(idx->dtype, idx->emb, queries, s, none, scratch, grid, &lists, st)
                 : launch_tc_search(idx->emb, queries, s, none, plan, scratch, idx->dev_err, &lists, st);
   if (e != cudaSuccess) return cuda_fail(e, "search kernel");
+  note_launch(idx, path, plan);
   e = launch_merge(lists, q, k, out_ids, out_scores, st);
   if (e != cudaSuccess) return cuda_fail(e, "merge kernel");
   idx->last_path = path;

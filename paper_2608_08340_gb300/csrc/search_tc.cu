@@ -49,7 +49,10 @@ bool make_map(CUtensorMap* m, const void* base, int64_t rows, int d, int box_row
 
 }  // namespace
 
-TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_stride) {
+int tc_pair_capacity() { return pair_capacity_query(); }
+
+TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_stride,
+               int force_pair, int pair_capacity) {
   TcPlan pl{};
   pl.qt = (s.q + kBlockM - 1) / kBlockM;
   int bn = 256;
@@ -62,50 +65,71 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
     if (units256 < 4LL * num_sms) bn = 128;
   }
   pl.block_n = bn;
+  // CTA pairs cut the operand bytes each SM loads per MMA by a third; they
+  // need 256-row corpus tiles and a device that fits clusters of two.  They
+  // run only on request: measured on GB300 they are no faster than single
+  // CTAs (the stage rate is the same; the epilogue and the copy/MMA overlap,
+  // not operand bytes, bound the kernel).
+  const bool pair = bn == 256 && pair_capacity > 0 && force_pair == 2;
+  pl.pair = pair ? 2 : 1;
+  pl.uqt = pair ? (pl.qt + 1) / 2 : pl.qt;
   pl.tile_stride = tile_stride < 1 ? 1 : tile_stride;
   const int64_t all_tiles = (s.n + bn - 1) / bn;
   pl.nt = static_cast<int>((all_tiles + pl.tile_stride - 1) / pl.tile_stride);
-  const int64_t units = static_cast<int64_t>(pl.nt) * pl.qt;
-  pl.grid = static_cast<int>(units < num_sms ? units : num_sms);
-  if (pl.grid < 1) pl.grid = 1;
+  const int64_t units = static_cast<int64_t>(pl.nt) * pl.uqt;
+  const int slots = pair ? pair_capacity : num_sms;     // schedule units in flight
+  int C = static_cast<int>(units < slots ? units : slots);
+  if (C < 1) C = 1;
+  pl.grid = C * pl.pair;
   // Windows of about 32 MB of corpus (one window when the corpus is small).
   const int64_t tile_bytes = static_cast<int64_t>(bn) * s.d * 2;
   const int64_t corpus = tile_bytes * pl.nt;
   pl.win = corpus <= (int64_t(80) << 20)
                ? pl.nt
                : static_cast<int>(std::max<int64_t>(1, (int64_t(32) << 20) / tile_bytes));
-  // Exact per-tile range of CTAs, by replaying the schedule of UnitSeq.
-  const int C = pl.grid;
+  // Exact per-tile range of schedule slots (CTAs or pairs), by replaying
+  // the schedule of UnitSeq.
   int per_tile = 1;
-  std::vector<int> hi(pl.qt, -1);
+  std::vector<int> hi(pl.uqt, -1);
   bool ok = true;
   for (int w = 0; static_cast<int64_t>(w) * pl.win < pl.nt; ++w) {
     const int tw = std::min(pl.win, pl.nt - w * pl.win);
-    const int64_t uw = static_cast<int64_t>(pl.qt) * tw;
+    const int64_t uw = static_cast<int64_t>(pl.uqt) * tw;
     for (int c = 0; c < C; ++c) {
       const int64_t l0 = uw * c / C, l1 = uw * (c + 1) / C;
       if (l0 >= l1) continue;
       for (int64_t j = l0 / tw; j <= (l1 - 1) / tw; ++j) {
-        if (c < first_cta(static_cast<int>(j), pl.qt, C)) ok = false;
+        if (c < first_cta(static_cast<int>(j), pl.uqt, C)) ok = false;
         hi[j] = std::max(hi[j], c);
       }
     }
   }
-  for (int j = 0; j < pl.qt; ++j)
-    per_tile = std::max(per_tile, hi[j] - first_cta(j, pl.qt, C) + 1);
-  if (!ok) per_tile = C;  // not expected; every CTA then gets a slot per tile
+  for (int j = 0; j < pl.uqt; ++j)
+    per_tile = std::max(per_tile, hi[j] - first_cta(j, pl.uqt, C) + 1);
+  if (!ok) per_tile = C;  // not expected; every slot then gets a list per tile
   pl.pmax = per_tile * epi_sets(list_len_for(s.k));
-  pl.stages = bn == 128 ? stages_for<128>() : stages_for<256>();
   const int K = list_len_for(s.k);
-  pl.smem = bn == 128 ? (K <= 16 ? smem_for<128, 16>() : smem_for<128, 32>())
-                      : (K <= 16 ? smem_for<256, 16>() : smem_for<256, 32>());
+  if (pair) {
+    pl.stages = stages_for<256, true>();
+    pl.smem = K <= 16 ? smem_for<256, 16, true>() : smem_for<256, 32, true>();
+  } else {
+    pl.stages = bn == 128 ? stages_for<128>() : stages_for<256>();
+    pl.smem = bn == 128 ? (K <= 16 ? smem_for<128, 16>() : smem_for<128, 32>())
+                        : (K <= 16 ? smem_for<256, 16>() : smem_for<256, 32>());
+  }
   return pl;
+}
+
+// List rows: one per (query tile, producer, query row); pair mode covers
+// 2 * uqt tiles (an odd qt leaves the last pair's second tile empty).
+static size_t list_rows(const TcPlan& pl) {
+  return static_cast<size_t>(pl.uqt) * pl.pair * pl.pmax * kBlockM;
 }
 
 size_t tc_scratch_bytes(const SearchShape& s, const TcPlan& pl) {
   const int K = list_len_for(s.k);
   const int stride = K > 32 ? 2 * K : K;
-  const size_t rows = static_cast<size_t>(pl.qt) * pl.pmax * kBlockM;
+  const size_t rows = list_rows(pl);
   size_t bytes = rows * stride * sizeof(uint64_t);
   if (K > 32) bytes += rows * (sizeof(uint64_t) + sizeof(int));
   return bytes;
@@ -113,23 +137,27 @@ size_t tc_scratch_bytes(const SearchShape& s, const TcPlan& pl) {
 
 cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s, const Fusion& fu,
                              const TcPlan& pl, void* scratch, int* dev_err, ListSet* lists,
-                             cudaStream_t st, const float* init_floor) {
+                             cudaStream_t st, const float* init_floor, uint64_t* qfloor,
+                             uint32_t gen) {
   CUtensorMap mq, me;
   // With a single query tile only its real rows are loaded (the remaining
   // rows of the A tile hold stale data whose TMEM lanes the epilogue never
   // reads); rows are loaded in multiples of 8, the swizzle atom height.
-  const int a_rows = pl.qt == 1 ? std::min(kBlockM, (s.q + 7) / 8 * 8) : kBlockM;
-  if (!make_map(&mq, Q, s.q, s.d, a_rows) || !make_map(&me, E, s.n, s.d, pl.block_n))
+  // Pair mode: each CTA loads all 128 rows of its tile and half of the
+  // corpus tile.
+  const int a_rows = pl.qt == 1 && pl.pair == 1 ? std::min(kBlockM, (s.q + 7) / 8 * 8) : kBlockM;
+  if (!make_map(&mq, Q, s.q, s.d, a_rows) ||
+      !make_map(&me, E, s.n, s.d, pl.block_n / pl.pair))
     return cudaErrorInvalidValue;
   const int K = list_len_for(s.k);
   const int stride = K > 32 ? 2 * K : K;
-  const size_t rows = static_cast<size_t>(pl.qt) * pl.pmax * kBlockM;
+  const size_t rows = list_rows(pl);
   TcParams prm{};
   prm.n = s.n;
   prm.d = s.d;
   prm.q = s.q;
   prm.k = s.k;
-  prm.qt = pl.qt;
+  prm.qt = pl.uqt;
   prm.nt = pl.nt;
   prm.win = pl.win;
   prm.pmax = pl.pmax;
@@ -142,15 +170,23 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
   prm.meta_worst = prm.lists + rows * stride;
   prm.meta_count = reinterpret_cast<int*>(prm.meta_worst + (K > 32 ? rows : 0));
   prm.dev_err = dev_err;
+  prm.qfloor = K <= 32 ? qfloor : nullptr;
+  prm.gen = gen;
   lists->keys = prm.lists;
   lists->P = pl.pmax;
   lists->TH = kBlockM;
   lists->stride = stride;
-  lists->C = pl.grid;
-  lists->qt = pl.qt;
+  lists->C = pl.grid / pl.pair;
+  lists->qt = pl.uqt;
   lists->sets = epi_sets(K);
   lists->klen = K;
+  lists->pair = pl.pair;
   const bool hybrid = fu.bm25 != nullptr;
+  if (pl.pair == 2) {
+    if (pl.block_n != 256) return cudaErrorInvalidValue;
+    return hybrid ? launch_pair256_fused(mq, me, prm, pl.grid, st)
+                  : launch_pair256_dense(mq, me, prm, pl.grid, st);
+  }
   if (pl.block_n == 128) return launch_bn128(mq, me, prm, pl.grid, hybrid, st);
   return hybrid ? launch_bn256_fused(mq, me, prm, pl.grid, st)
                 : launch_bn256_dense(mq, me, prm, pl.grid, st);

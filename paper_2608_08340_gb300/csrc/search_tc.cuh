@@ -64,6 +64,11 @@ struct TcParams {
   int* meta_count;      // buffered lists: kept keys per (list, row)
   uint64_t* meta_worst; // buffered lists: K-th key per (list, row)
   int* dev_err;
+  // Optional (register lists only): per query, a lower bound of its k-th best
+  // score shared by every list of the search, tagged with `gen` (entries of
+  // other searches read as -inf); see shared_floor_read.
+  uint64_t* qfloor;
+  uint32_t gen;
 };
 
 // Units of one CTA in processing order.  The corpus tiles are cut into
@@ -117,18 +122,27 @@ __host__ __device__ __forceinline__ int first_cta(int j, int qt, int C) {
   return c < 0 ? 0 : c;
 }
 
-template <int BN>
+// Corpus rows one CTA loads per stage: BN, or BN / 2 when a CTA pair shares
+// the tile (each CTA of the pair loads half of its rows).
+template <int BN, bool kPair>
+constexpr uint32_t b_stage_bytes() {
+  return static_cast<uint32_t>(kPair ? BN / 2 : BN) * 128;
+}
+
+template <int BN, bool kPair = false>
 constexpr int stages_for() {
-  return kSmemBudget / (kAStageBytes + BN * 128) > 8 ? 8 : kSmemBudget / (kAStageBytes + BN * 128);
+  return kSmemBudget / (kAStageBytes + b_stage_bytes<BN, kPair>()) > 8
+             ? 8
+             : kSmemBudget / (kAStageBytes + b_stage_bytes<BN, kPair>());
 }
 
 // Per epilogue thread: one 32-float row where a chunk's scores are staged so
 // that candidate columns can be read back by index.
 constexpr int kStageRowBytes = 32 * 4;
 
-template <int BN, int K>
+template <int BN, int K, bool kPair = false>
 constexpr size_t smem_for() {
-  return static_cast<size_t>(stages_for<BN>()) * (kAStageBytes + BN * 128) +
+  return static_cast<size_t>(stages_for<BN, kPair>()) * (kAStageBytes + b_stage_bytes<BN, kPair>()) +
          static_cast<size_t>(epi_sets(K)) * 128 * kStageRowBytes + 1024 + 256;
 }
 
@@ -203,6 +217,94 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar) {
       : "memory");
 }
 
+// ----------------------------------------------------------- CTA pairs
+// A cluster of two CTAs can issue one MMA with M = 256 (cta_group::2): each
+// CTA holds 128 rows of A and half of the N rows of B in its own shared
+// memory at the same offsets, and each CTA's TMEM receives the 128 x N
+// accumulator of its own A rows.  Rank 0 of the pair issues the MMAs.  A
+// kernel uses one cta_group for all of its tcgen05 instructions.
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ uint32_t cluster_index() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+  return r;
+}
+
+// Every thread of both CTAs; orders shared-memory writes before the barrier
+// with reads after it across the cluster.
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+}
+
+// Address of the same shared-memory variable in the CTA of cluster rank `rank`.
+__device__ __forceinline__ uint32_t cluster_addr(const void* p, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr(p)), "r"(rank));
+  return r;
+}
+
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t caddr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(caddr)
+               : "memory");
+}
+
+// TMA load into this CTA's shared memory whose completion is counted on an
+// mbarrier of either CTA of the pair (cluster address).
+__device__ __forceinline__ void tma_load_2d_pair(void* dst, const CUtensorMap* map, uint32_t bar_caddr,
+                                                 int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.cta_group::2"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_addr(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_caddr), "r"(x), "r"(y)
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t* slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                   smem_addr(slot)),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+
+__device__ __forceinline__ void mma_bf16_pair(uint32_t d_tmem, uint64_t a, uint64_t b,
+                                              uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrives once on the mbarrier at this offset in every CTA of `mask` when the
+// pair's MMAs issued so far have completed.
+__device__ __forceinline__ void mma_commit_pair_mc(uint64_t* bar, uint16_t mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(smem_addr(bar)),
+      "h"(mask)
+      : "memory");
+}
+
+__device__ __forceinline__ void mma_commit_pair(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_addr(bar))
+      : "memory");
+}
+
 // Issues a 32-column TMEM load (32 lanes x 32 columns of 32 bits); the
 // registers are valid only after tmem_wait_ld() on the same array.
 __device__ __forceinline__ void tmem_ld32_async(uint32_t taddr, uint32_t (&r)[32]) {
@@ -232,16 +334,73 @@ __device__ __forceinline__ void tmem_wait_ld(uint32_t (&r)[32]) {
                : "memory");
 }
 
-// max of 32 values, depth-5 tree.
+// ------------------------------------------------------- shared k-th floors
+// Every list that holds k scores >= f proves that the query's k-th best score
+// is >= f, so any list may drop scores below f.  Lists publish such bounds per
+// query with a 64-bit atomic max of (gen << 32 | order-preserving bits of f)
+// and read the current value before each unit; an entry of another search
+// (other gen) reads as -inf, so the array never needs clearing.
+__device__ __forceinline__ uint32_t ordered_bits(float f) {
+  const uint32_t b = __float_as_uint(f);
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+__device__ __forceinline__ float from_ordered_bits(uint32_t o) {
+  return __uint_as_float((o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o);
+}
+
+__device__ __forceinline__ float shared_floor_read(const uint64_t* qf, int64_t qi, uint32_t gen) {
+  const unsigned long long v = __ldcg(reinterpret_cast<const unsigned long long*>(qf + qi));
+  return static_cast<uint32_t>(v >> 32) == gen ? from_ordered_bits(static_cast<uint32_t>(v))
+                                               : -INFINITY;
+}
+
+__device__ __forceinline__ void shared_floor_raise(uint64_t* qf, int64_t qi, uint32_t gen, float f) {
+  atomicMax(reinterpret_cast<unsigned long long*>(qf + qi),
+            (static_cast<unsigned long long>(gen) << 32) | ordered_bits(f));
+}
+
+// Sorts 32 values descending in registers (bitonic network, 240 exchanges);
+// the stages are template instances so that every index is a constant.
+template <int KS, int JS>
+__device__ __forceinline__ void bitonic_stage32(float (&a)[32]) {
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    const int l = i ^ JS;
+    if (l > i) {
+      const float hi = fmaxf(a[i], a[l]), lo = fminf(a[i], a[l]);
+      const bool desc = (i & KS) == 0;
+      a[i] = desc ? hi : lo;
+      a[l] = desc ? lo : hi;
+    }
+  }
+  if constexpr (JS > 1) bitonic_stage32<KS, JS / 2>(a);
+}
+
+template <int KS = 2>
+__device__ __forceinline__ void bitonic_desc32(float (&a)[32]) {
+  bitonic_stage32<KS, KS / 2>(a);
+  if constexpr (KS < 32) bitonic_desc32<KS * 2>(a);
+}
+
+// Three-input maximum (one instruction on sm_100 and later).
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
+// max of 32 values: 16 three- and two-input maxima (the epilogue's filter runs
+// this once per 32 scores, so its instruction count bounds the epilogue).
 __device__ __forceinline__ float max32(const float (&v)[32]) {
-  float a[16];
+  float a[12];
 #pragma unroll
-  for (int i = 0; i < 16; ++i) a[i] = fmaxf(v[2 * i], v[2 * i + 1]);
-#pragma unroll
-  for (int w = 8; w >= 1; w >>= 1)
-#pragma unroll
-    for (int i = 0; i < w; ++i) a[i] = fmaxf(a[2 * i], a[2 * i + 1]);
-  return a[0];
+  for (int i = 0; i < 10; ++i) a[i] = fmax3(v[3 * i], v[3 * i + 1], v[3 * i + 2]);
+  a[10] = v[30];
+  a[11] = v[31];
+  const float b0 = fmax3(a[0], a[1], a[2]), b1 = fmax3(a[3], a[4], a[5]);
+  const float b2 = fmax3(a[6], a[7], a[8]), b3 = fmax3(a[9], a[10], a[11]);
+  return fmaxf(fmax3(b0, b1, b2), b3);
 }
 
 // Waits without looking at the abort word (used to drain in-flight copies and
@@ -278,6 +437,7 @@ struct EpiList<K, false> {
   __device__ __forceinline__ float floor() const { return t.floor; }
   __device__ __forceinline__ void push(float s, uint32_t id) { t.push(s, id); }
   __device__ __forceinline__ void insert(float s, uint32_t id) { t.insert(s, id); }
+  __device__ __forceinline__ float kth(int k) const { return t.kth(k); }
   __device__ __forceinline__ void sync(bool, bool) {}
   __device__ __forceinline__ void finalize(const TcParams&, int64_t, bool) {}
 };
@@ -325,12 +485,18 @@ struct EpiList<K, true> {
 
 // ----------------------------------------------------------------- kernel
 
-template <int BN, int K, bool kHybrid>
+// kPair: the grid is made of clusters of two CTAs that share every unit: a
+// unit covers query tiles 2J and 2J + 1 (one per CTA) and corpus tile t of BN
+// rows (BN / 2 loaded by each CTA); rank 0 issues M = 256 MMAs for both.  Per
+// MMA each CTA then reads 128 x 16 + BN / 2 x 16 operand elements instead of
+// 128 x 16 + BN x 16.  The unit sequence (UnitSeq) runs over pairs: p.qt
+// counts pairs of query tiles and the pair index plays the CTA index.
+template <int BN, int K, bool kHybrid, bool kPair = false>
 __global__ void __launch_bounds__(threads_for(K), 1)
 tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_e,
                  const TcParams p) {
-  constexpr int S = stages_for<BN>();
-  constexpr uint32_t kBStageBytes = BN * 128;
+  constexpr int S = stages_for<BN, kPair>();
+  constexpr uint32_t kBStageBytes = b_stage_bytes<BN, kPair>();
   constexpr uint32_t kTmemCols = 2 * BN;
   constexpr int kEpiSets = epi_sets(K);
   extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -348,7 +514,19 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int cta = blockIdx.x, C = gridDim.x;
+  // Pair mode: rank 0 of each cluster is the leader (issues the MMAs, owns
+  // the full / tempty / mma_done barriers that count both CTAs).
+  const uint32_t rank = kPair ? cluster_rank() : 0u;
+  const bool leader = rank == 0;
+  const int cta = kPair ? static_cast<int>(cluster_index()) : static_cast<int>(blockIdx.x);
+  const int C = kPair ? static_cast<int>(gridDim.x) / 2 : static_cast<int>(gridDim.x);
+  // Bytes one stage brings into the leader's full barrier (both CTAs in pair mode).
+  const uint32_t stage_tx = (p.a_bytes + kBStageBytes) * (kPair ? 2u : 1u);
+  // Row coordinates of this CTA's part of unit (J, t).
+  auto a_row = [&](int J) { return (kPair ? 2 * J + static_cast<int>(rank) : J) * kBlockM; };
+  auto b_row = [&](int t) {
+    return t * BN + (kPair ? static_cast<int>(rank) * (BN / 2) : 0);
+  };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S; ++s) {
@@ -357,7 +535,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
-      mbar_init(&tempty[b], 4);
+      mbar_init(&tempty[b], kPair ? 8 : 4);   // four epilogue warps per CTA
     }
     mbar_init(mma_done, 1);
     *abort_flag = 0;
@@ -365,23 +543,36 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     prefetch_map(&map_q);
     prefetch_map(&map_e);
   }
+  // The peer's copies and arrivals target the leader's barriers: both CTAs'
+  // barriers are initialised before either CTA issues anything.
+  if constexpr (kPair) cluster_sync();
+  auto load_stage = [&](int s, int kb, int J, int t) {
+    if (kPair) {
+      if (leader) mbar_arrive_expect_tx(&full[s], stage_tx);
+      const uint32_t bar = cluster_addr(&full[s], 0);                  // the leader's full[s]
+      tma_load_2d_pair(sA + s * kAStageBytes, &map_q, bar, kb * kBlockK, a_row(J));
+      tma_load_2d_pair(sB + s * kBStageBytes, &map_e, bar, kb * kBlockK, b_row(t));
+    } else {
+      mbar_arrive_expect_tx(&full[s], stage_tx);
+      tma_load_2d(sA + s * kAStageBytes, &map_q, &full[s], kb * kBlockK, a_row(J));
+      tma_load_2d(sB + s * kBStageBytes, &map_e, &full[s], kb * kBlockK, b_row(t));
+    }
+  };
   int pre_issued = 0;           // stages the producer issued before the setup barrier
   if (threadIdx.x == 0) {
     // The ring is empty: start the first loads while TMEM is being allocated.
     UnitSeq us;
     us.start(p, cta, C);
     for (; us.valid() && pre_issued < S; us.next()) {
-      for (int kb = 0; kb < p.kblocks && pre_issued < S; ++kb, ++pre_issued) {
-        mbar_arrive_expect_tx(&full[pre_issued], p.a_bytes + kBStageBytes);
-        tma_load_2d(sA + pre_issued * kAStageBytes, &map_q, &full[pre_issued], kb * kBlockK,
-                    us.j() * kBlockM);
-        tma_load_2d(sB + pre_issued * kBStageBytes, &map_e, &full[pre_issued], kb * kBlockK,
-                    us.t() * BN);
-      }
+      for (int kb = 0; kb < p.kblocks && pre_issued < S; ++kb, ++pre_issued)
+        load_stage(pre_issued, kb, us.j(), us.t());
       if (pre_issued >= S) break;
     }
   }
-  if (warp == 1) tmem_alloc(tmem_slot, kTmemCols);
+  if (warp == 1) {
+    if constexpr (kPair) tmem_alloc_pair(tmem_slot, kTmemCols);
+    else tmem_alloc(tmem_slot, kTmemCols);
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -411,22 +602,22 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             continue;
           }
           if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, p.dev_err)) { ok = false; break; }
-          mbar_arrive_expect_tx(&full[s], p.a_bytes + kBStageBytes);
-          tma_load_2d(sA + s * kAStageBytes, &map_q, &full[s], kb * kBlockK, j * kBlockM);
-          tma_load_2d(sB + s * kBStageBytes, &map_e, &full[s], kb * kBlockK, t * BN);
+          load_stage(s, kb, j, t);
           issued |= 1u << s;
           parity = (parity & ~(1u << s)) | (ph << s);
           if (++s == S) { s = 0; ph ^= 1u; }
         }
       }
-      for (int i = 0; i < S; ++i)
-        if (issued & (1u << i)) mbar_drain(&full[i], (parity >> i) & 1u, p.dev_err);
+      // The leader's full barriers also count the peer's copies.
+      if (leader)
+        for (int i = 0; i < S; ++i)
+          if (issued & (1u << i)) mbar_drain(&full[i], (parity >> i) & 1u, p.dev_err);
     }
     __syncwarp();
   } else if (warp == 1) {
-    if (lane == 0) {
+    if (lane == 0 && leader) {
       // ------------------------------------------------ MMA issuer
-      constexpr uint32_t idesc = idesc_bf16(kBlockM, BN);
+      constexpr uint32_t idesc = idesc_bf16(kPair ? 2 * kBlockM : kBlockM, BN);
       int s = 0;
       uint32_t ph = 0;
       int acc = 0;
@@ -434,7 +625,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       bool ok = true;
       UnitSeq us;
       for (us.start(p, cta, C); ok && us.valid(); us.next()) {
-        if (!mbar_wait(&tempty[acc], acc_ph ^ 1u, abort_flag, p.dev_err)) break;
+        if (!mbar_wait<kPair>(&tempty[acc], acc_ph ^ 1u, abort_flag, p.dev_err)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
         for (int kb = 0; kb < p.kblocks; ++kb) {
@@ -442,17 +633,26 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
           tc_fence_after();
           const uint64_t a = sw128_desc(smem_addr(sA + s * kAStageBytes));
           const uint64_t b = sw128_desc(smem_addr(sB + s * kBStageBytes));
+          if constexpr (kPair) {
 #pragma unroll
-          for (int kk = 0; kk < kBlockK / kUmmaK; ++kk)
-            mma_bf16(d_tmem, a + 2 * kk, b + 2 * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
-          mma_commit(&empty[s]);
+            for (int kk = 0; kk < kBlockK / kUmmaK; ++kk)
+              mma_bf16_pair(d_tmem, a + 2 * kk, b + 2 * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
+            mma_commit_pair_mc(&empty[s], 0x3);
+          } else {
+#pragma unroll
+            for (int kk = 0; kk < kBlockK / kUmmaK; ++kk)
+              mma_bf16(d_tmem, a + 2 * kk, b + 2 * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
+            mma_commit(&empty[s]);
+          }
           if (++s == S) { s = 0; ph ^= 1u; }
         }
         if (!ok) break;
-        mma_commit(&tfull[acc]);
+        if constexpr (kPair) mma_commit_pair_mc(&tfull[acc], 0x3);
+        else mma_commit(&tfull[acc]);
         if (++acc == 2) { acc = 0; acc_ph ^= 1u; }
       }
-      mma_commit(mma_done);
+      if constexpr (kPair) mma_commit_pair(mma_done);
+      else mma_commit(mma_done);
       mbar_drain(mma_done, 0, p.dev_err);
     }
     __syncwarp();
@@ -464,21 +664,25 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     const int set = (warp - 2) >> 2;
     const int eg = warp & 3;                 // TMEM lane group of this warp
     const int row = eg * 32 + lane;          // query row within a tile
-    const int per_tile = p.pmax / kEpiSets;  // CTAs per query tile with a list slot
-    auto list_row = [&](int j) -> int64_t {
-      const int pc = cta - first_cta(j, p.qt, C);
-      return (static_cast<int64_t>(j) * p.pmax + pc * kEpiSets + set) * kBlockM + row;
+    const int per_tile = p.pmax / kEpiSets;  // CTAs (pairs) per unit query tile with a list slot
+    // Unit query tile J covers this CTA's query tile qtile(J) (one of a pair's two).
+    auto qtile = [&](int J) { return kPair ? 2 * J + static_cast<int>(rank) : J; };
+    auto list_row = [&](int J) -> int64_t {
+      const int pc = cta - first_cta(J, p.qt, C);
+      return (static_cast<int64_t>(qtile(J)) * p.pmax + pc * kEpiSets + set) * kBlockM + row;
     };
-    auto owns = [&](int j) {
-      const int pc = cta - first_cta(j, p.qt, C);
+    auto owns = [&](int J) {
+      const int pc = cta - first_cta(J, p.qt, C);
       return pc >= 0 && pc < per_tile;
     };
     EpiList<K> list;
     list.clear();
 
-    // This CTA owns the list slots (j, cta - first_cta(j)); empty them first.
-    for (int j = 0; j < p.qt; ++j)
-      if (owns(j) && j * kBlockM + row < p.q) list.init_mem(p, list_row(j), j * kBlockM + row);
+    // This CTA owns the list slots (J, cta - first_cta(J)); empty them first.
+    for (int J = 0; J < p.qt; ++J) {
+      const int qi = qtile(J) * kBlockM + row;
+      if (owns(J) && qi < p.q) list.init_mem(p, list_row(J), qi);
+    }
 
     int cur_j = -1;
     int64_t cur_sr = 0;
@@ -489,22 +693,27 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     for (us.start(p, cta, C); us.valid(); us.next(), ++seq) {
       if (seq % kEpiSets != set) continue;
       const int acc = seq & 1;
-      const int j = us.j();
+      const int J = us.j();
+      const int j = qtile(J);                // this CTA's query tile
       const int64_t t = us.t();
       const bool valid = j * kBlockM + row < p.q;
       const bool warp_live = j * kBlockM + eg * 32 < p.q;
-      if (j != cur_j) {
+      if (J != cur_j) {
         if (cur_j >= 0 && cur_valid) list.save(p, cur_sr);
-        if (!owns(j)) {              // cannot happen when the host plan holds
+        if (!owns(J)) {              // cannot happen when the host plan holds
           atomicExch(p.dev_err, 2);
           *abort_flag = 1;
         }
-        cur_j = j;
-        cur_sr = list_row(j);
-        cur_valid = valid && owns(j);
+        cur_j = J;
+        cur_sr = list_row(J);
+        cur_valid = valid && owns(J);
         if (cur_valid) list.load(p, cur_sr); else list.clear();
       }
       const bool act = cur_valid;
+      // Shared bound of this query's k-th best score, read while the MMAs run.
+      float gfl = -INFINITY;
+      if (K <= 32 && p.qfloor != nullptr && act)
+        gfl = shared_floor_read(p.qfloor, static_cast<int64_t>(j) * kBlockM + row, p.gen);
       if (!mbar_wait(&tfull[acc], (acc_ph >> acc) & 1u, abort_flag, p.dev_err)) break;
       tc_fence_after();
       if (warp_live) {
@@ -591,63 +800,146 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         float bound = -INFINITY;
         if constexpr (K <= 32) {
           if (__any_sync(0xffffffffu, act && !list.full())) {
-          // A list that is not full yet would take almost every score of this
-          // unit as a candidate.  Cut the unit into K groups of BN / K
-          // scores: each group holds a score >= its maximum, so the smallest
-          // group maximum is <= the unit's K-th best score and nothing below
-          // it can enter the list.
-          constexpr int G = K / NC;           // groups per chunk
-          static_assert(G >= 1 && 32 % G == 0, "group layout");
-          float gmin = INFINITY;
+            // A list that is not full yet would take almost every score of
+            // this unit as a candidate.  Cut the unit's columns into groups:
+            // the k-th largest group maximum is reached by k distinct scores
+            // of the unit, so it is <= the unit's k-th best score, and no
+            // score below it can be among the query's k best.  Lists of 16
+            // or 32 use 32 groups and sort their maxima (a tight bound pays
+            // for the sort when each insertion costs 16-32 steps); lists of
+            // 8 use K groups and the smallest maximum, which needs no sort.
+            if constexpr (K <= 8) {
+              constexpr int G = K / NC;         // groups per 32-column chunk
+              static_assert(G >= 1 && 32 % G == 0, "group layout");
+              float gmin = INFINITY;
 #pragma unroll 1
-          for (int c = 0; c < NC; ++c) {
-            __syncwarp();
-            tmem_ld32_async(taddr + c * 32, ra);
-            tmem_wait_ld(ra);
-            float v[32];
-            scores(ra, c, v);
+              for (int c = 0; c < NC; ++c) {
+                __syncwarp();
+                tmem_ld32_async(taddr + c * 32, ra);
+                tmem_wait_ld(ra);
+                float v[32];
+                scores(ra, c, v);
 #pragma unroll
-            for (int g = 0; g < G; ++g) {
-              float m = v[g * (32 / G)];
+                for (int g = 0; g < G; ++g) {
+                  constexpr int L = 32 / G;
+                  float m = v[g * L];
 #pragma unroll
-              for (int i = 1; i < 32 / G; ++i) m = fmaxf(m, v[g * (32 / G) + i]);
-              gmin = fminf(gmin, m);
+                  for (int i = 1; i + 1 < L; i += 2) m = fmax3(m, v[g * L + i], v[g * L + i + 1]);
+                  if constexpr (L % 2 == 0) m = fmaxf(m, v[g * L + L - 1]);
+                  gmin = fminf(gmin, m);
+                }
+              }
+              bound = gmin;
+            } else {
+            constexpr int GPC = 32 / NC;        // groups per 32-column chunk
+            constexpr int L = 32 / GPC;         // columns per group
+            static_assert(GPC * NC == 32 && L >= 2, "group layout");
+            float gm[32];
+#pragma unroll
+            for (int c = 0; c < NC; ++c) {
+              __syncwarp();
+              tmem_ld32_async(taddr + c * 32, ra);
+              tmem_wait_ld(ra);
+              float v[32];
+              scores(ra, c, v);
+#pragma unroll
+              for (int g = 0; g < GPC; ++g) {
+                float m = v[g * L];
+#pragma unroll
+                for (int i = 1; i + 1 < L; i += 2) m = fmax3(m, v[g * L + i], v[g * L + i + 1]);
+                if constexpr (L % 2 == 0) m = fmaxf(m, v[g * L + L - 1]);
+                gm[c * GPC + g] = m;
+              }
+            }
+            bitonic_desc32(gm);
+            const int kk = p.k < 32 ? p.k : 32;
+            bound = reg_select(gm, kk - 1);
             }
           }
-          bound = gmin;
-          }
         }
+        const float lb = fmaxf(bound, gfl);     // admission bound of this unit
         __syncwarp();
         tmem_ld32_async(taddr, ra);
 #pragma unroll 1
         for (int c = 0; c < NC; c += 2) {
           tmem_wait_ld(ra);
           tmem_ld32_async(taddr + (c + 1) * 32, rb);
-          process(ra, c, bound);
+          process(ra, c, lb);
           tmem_wait_ld(rb);
           if (c + 2 < NC) tmem_ld32_async(taddr + (c + 2) * 32, ra);
-          process(rb, c + 1, bound);
+          process(rb, c + 1, lb);
+        }
+        if constexpr (K <= 32) {
+          // Publish what this list now proves about the query's k-th best.
+          if (p.qfloor != nullptr && act) {
+            const float pub = fmaxf(list.kth(p.k), bound);
+            if (pub > gfl)
+              shared_floor_raise(p.qfloor, static_cast<int64_t>(j) * kBlockM + row, p.gen, pub);
+          }
         }
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty[acc]);
+      if (lane == 0) {
+        // Pair mode: the epilogue warps of both CTAs release the accumulator
+        // at the leader.
+        if constexpr (kPair) mbar_arrive_cluster(cluster_addr(&tempty[acc], 0));
+        else mbar_arrive(&tempty[acc]);
+      }
       acc_ph ^= 1u << acc;
     }
     if (cur_j >= 0 && cur_valid) list.save(p, cur_sr);
     if (K > 32) {
-      for (int j = 0; j < p.qt; ++j)
-        if (owns(j)) list.finalize(p, list_row(j), j * kBlockM + row < p.q);
+      for (int J = 0; J < p.qt; ++J)
+        if (owns(J)) list.finalize(p, list_row(J), qtile(J) * kBlockM + row < p.q);
     }
   }
 
   tc_fence_before();
-  __syncthreads();
+  // Pair mode: neither CTA leaves (or frees TMEM) while the other may still
+  // signal its barriers; the leader's MMAs have drained (mma_done) by now.
+  if constexpr (kPair) cluster_sync();
+  else __syncthreads();
   tc_fence_after();
-  if (warp == 1) tmem_dealloc(tmem_base, kTmemCols);
+  if (warp == 1) {
+    if constexpr (kPair) tmem_dealloc_pair(tmem_base, kTmemCols);
+    else tmem_dealloc(tmem_base, kTmemCols);
+  }
 }
 
 // ----------------------------------------------------------------- launch
+
+// Pair mode: clusters of two CTAs; `grid` counts CTAs (even).
+template <int BN, int K, bool H>
+cudaError_t launch_pair_variant(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
+                                int grid, cudaStream_t st) {
+  constexpr size_t smem = smem_for<BN, K, true>();
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(tc_search_kernel<BN, K, H, true>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(threads_for(K));
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, tc_search_kernel<BN, K, H, true>, mq, me, prm);
+}
+
+// Clusters of two CTAs of a pair-mode search kernel that fit on the device at
+// once (the kernels' shared-memory use keeps one CTA per SM).
+int pair_capacity_query();
 
 template <int BN, int K, bool H>
 cudaError_t launch_variant(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
@@ -691,6 +983,10 @@ cudaError_t launch_bn256_dense(const CUtensorMap& mq, const CUtensorMap& me, con
                                int grid, cudaStream_t st);
 cudaError_t launch_bn256_fused(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
                                int grid, cudaStream_t st);
+cudaError_t launch_pair256_dense(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
+                                 int grid, cudaStream_t st);
+cudaError_t launch_pair256_fused(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
+                                 int grid, cudaStream_t st);
 
 }  // namespace tc
 }  // namespace oprag

@@ -8,6 +8,8 @@ from __future__ import annotations
 
 import ctypes
 
+_I32 = ctypes.c_int32
+
 import numpy as np
 import torch
 
@@ -163,6 +165,10 @@ class Index:
     def force_path(self, path: str | None) -> None:
         self.set_option(_lib.OPRAG_OPT_PATH, {None: 0, "simt": 1, "tc": 2}[path])
 
+    def force_pair(self, mode: str | None) -> None:
+        """None: automatic; "single": one CTA per MMA; "pair": CTA pairs."""
+        self.set_option(_lib.OPRAG_OPT_PAIR, {None: 0, "single": 1, "pair": 2}[mode])
+
     def force_block_n(self, bn: int | None) -> None:
         self.set_option(_lib.OPRAG_OPT_BLOCK_N, bn or 0)
 
@@ -175,6 +181,15 @@ class Index:
         check(self._lib.oprag_index_last_timing(self._h, ctypes.byref(a), ctypes.byref(b),
                                                 ctypes.byref(c)))
         return {"lexical_ms": a.value, "search_ms": b.value, "merge_ms": c.value}
+
+    @property
+    def last_launch(self) -> dict:
+        """Main kernel launch of the last search: grid (CTAs), cluster (2 = CTA
+        pairs), block_n; zeros for the SIMT kernel."""
+        g, c, b = _I32(), _I32(), _I32()
+        check(self._lib.oprag_index_last_launch(self._h, ctypes.byref(g), ctypes.byref(c),
+                                                ctypes.byref(b)))
+        return {"grid": g.value, "cluster": c.value, "block_n": b.value}
 
     @property
     def last_path(self) -> str:
