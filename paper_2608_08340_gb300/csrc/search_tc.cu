@@ -81,12 +81,17 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
   int C = static_cast<int>(units < slots ? units : slots);
   if (C < 1) C = 1;
   pl.grid = C * pl.pair;
-  // Windows of about 32 MB of corpus (one window when the corpus is small).
+  // Windows of about 32 MB of corpus.  Inside a window every CTA works on
+  // a contiguous share of (query tile, corpus tile) units, so at any moment
+  // the CTAs read tiles spread over the whole window: a window that stays in
+  // L2 is read from HBM about once.  With few query tiles the CTAs of
+  // one query tile already read the corpus in step, and one window over a
+  // small corpus (<= 80 MB) keeps the list count per query tile low (up to 8
+  // query tiles: measured, windows then cost more in lists than they save).
   const int64_t tile_bytes = static_cast<int64_t>(bn) * s.d * 2;
   const int64_t corpus = tile_bytes * pl.nt;
-  pl.win = corpus <= (int64_t(80) << 20)
-               ? pl.nt
-               : static_cast<int>(std::max<int64_t>(1, (int64_t(32) << 20) / tile_bytes));
+  const int win32 = static_cast<int>(std::max<int64_t>(1, (int64_t(32) << 20) / tile_bytes));
+  pl.win = corpus <= (int64_t(80) << 20) && pl.uqt <= 8 ? pl.nt : std::min(win32, pl.nt);
   // Exact per-tile range of schedule slots (CTAs or pairs), by replaying
   // the schedule of UnitSeq.
   int per_tile = 1;
