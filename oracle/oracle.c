@@ -11,8 +11,8 @@
  *
  * What each function follows:
  *   oracle_dense_scores  -- dense inner-product scoring of a query against
- *                           every chunk embedding ("vectorized matrix
- *                           operations over the embedding matrix", Sec. 4.4;
+ *                           every chunk embedding (the whole embedding
+ *                           matrix scored at once, Sec. 4.4;
  *                           vectors are L2-normalised by Op_embed, Sec. 4.3,
  *                           so inner product == cosine).
  *   oracle_search        -- TopK over the whole index, Sec. 3.2 (Op_retrieve,

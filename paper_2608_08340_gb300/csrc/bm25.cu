@@ -1,6 +1,6 @@
 // Lexical half of the hybrid search (Sec. 4.4): BM25 of every (query, chunk)
-// pair through inverted postings, which "visits only documents that contain
-// query terms while preserving exact full-corpus BM25 semantics".
+// pair through inverted postings, touching only the chunks that hold a query
+// term and giving the same scores as a scan of the whole corpus.
 //
 // The per-posting weight idf(t) * tf (k1 + 1) / (tf + k1 (1 - b + b |d| / avgdl))
 // does not depend on the query, so it is computed once on the host when the
@@ -9,10 +9,15 @@
 // list (a repeated term counts again).
 //
 // One CTA per (query, tile of 8192 chunks) accumulates those sums in shared
-// memory, one term at a time (the postings of one term hold each chunk at
-// most once, so the adds of a term never collide and the summation order is
-// fixed).  It writes the tile's row of the q x n BM25 matrix and folds the
-// tile maximum into the per-query maximum that normalises the lexical score.
+// memory, one term at a time in the query's order.  A dense term (held by
+// more than half of the chunks, stored as a row of weights with zeros where
+// absent) is added element-wise with 16-byte loads, each thread keeping the
+// same elements, so consecutive dense terms need no barrier; a sparse term
+// scatters its postings (each chunk at most once per term, so its adds never
+// collide).  Adding a zero weight leaves an fp32 sum unchanged, so both forms
+// give the same sums in the same order.  The CTA writes the tile's row of the
+// q x n BM25 matrix and folds the tile maximum into the per-query maximum
+// that normalises the lexical score.
 #include "common.cuh"
 #include "internal.h"
 
@@ -23,15 +28,17 @@ namespace {
 constexpr int kDocTile = 8192;
 constexpr int kBm25Threads = 256;
 constexpr int kTermsPerPass = kBm25Threads / 32;
+constexpr int kScatterUnroll = 4;      // postings loaded per thread before the adds
+constexpr int kSkipTerm = -2;          // term id outside the vocabulary
 
-// First position in [lo, hi) whose value is >= key (hi if none); the array is
+// First position in [lo, hi) whose chunk is >= key (hi if none); chunks are
 // ascending.  Warp-collective: 32 probes per round.
-__device__ int64_t warp_lower_bound(const int32_t* a, int64_t lo, int64_t hi, int32_t key) {
+__device__ int64_t warp_lower_bound(const int2* a, int64_t lo, int64_t hi, int32_t key) {
   const int lane = threadIdx.x & 31;
   while (hi - lo > 32) {
     const int64_t step = (hi - lo + 31) / 32;
     const int64_t pos = lo + lane * step;
-    const bool less = pos < hi && a[pos] < key;
+    const bool less = pos < hi && a[pos].x < key;
     const int c = __popc(__ballot_sync(0xffffffffu, less));
     if (c == 0) return lo;
     const int64_t next = lo + static_cast<int64_t>(c) * step;
@@ -39,7 +46,7 @@ __device__ int64_t warp_lower_bound(const int32_t* a, int64_t lo, int64_t hi, in
     if (c < 32 && next < hi) hi = next;
   }
   const int64_t pos = lo + lane;
-  const bool less = pos < hi && a[pos] < key;
+  const bool less = pos < hi && a[pos].x < key;
   return lo + __popc(__ballot_sync(0xffffffffu, less));
 }
 
@@ -47,48 +54,93 @@ __global__ void __launch_bounds__(kBm25Threads)
 bm25_matrix_kernel(SparseIndex sp, int64_t n, const int32_t* __restrict__ q_indptr,
                    const int32_t* __restrict__ q_terms, float* __restrict__ out, int64_t ld,
                    float* __restrict__ out_max) {
-  __shared__ float acc[kDocTile];
+  __shared__ __align__(16) float acc[kDocTile];
   __shared__ int64_t rng_lo[kTermsPerPass], rng_hi[kTermsPerPass];
+  __shared__ int slot_of[kTermsPerPass];
   __shared__ float red[kBm25Threads / 32];
   const int qi = blockIdx.x;
   const int64_t d0 = static_cast<int64_t>(blockIdx.y) * kDocTile;
   const int64_t d1 = min(n, d0 + kDocTile);
+  const int nv = static_cast<int>((d1 - d0 + 3) / 4);     // float4 groups of this tile
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float4* acc4 = reinterpret_cast<float4*>(acc);
 
-  for (int i = threadIdx.x; i < kDocTile; i += blockDim.x) acc[i] = 0.f;
+  for (int i = threadIdx.x; i < kDocTile / 4; i += blockDim.x) acc4[i] = make_float4(0.f, 0.f, 0.f, 0.f);
 
   const int t0 = q_indptr[qi], t1 = q_indptr[qi + 1];
+  bool pending = true;      // element-wise work since the last barrier came from a scatter
   for (int base = t0; base < t1; base += kTermsPerPass) {
-    // Locate each term's postings inside [d0, d1): one warp per term.
+    // Classify each term of the pass and locate a sparse term's postings
+    // inside [d0, d1): one warp per term.
     const int ti = base + warp;
     if (ti < t1) {
       const int32_t term = q_terms[ti];
+      int slot = kSkipTerm;
       int64_t lo = 0, hi = 0;
       if (term >= 0 && term < sp.vocab) {
-        const int64_t p0 = sp.post_ptr[term], p1 = sp.post_ptr[term + 1];
-        lo = warp_lower_bound(sp.post_doc, p0, p1, static_cast<int32_t>(d0));
-        hi = warp_lower_bound(sp.post_doc, lo, p1, static_cast<int32_t>(d1));
+        slot = sp.dense_slot[term];
+        if (slot < 0) {
+          const int64_t p0 = sp.post_ptr[term], p1 = sp.post_ptr[term + 1];
+          lo = warp_lower_bound(sp.post, p0, p1, static_cast<int32_t>(d0));
+          hi = warp_lower_bound(sp.post, lo, p1, static_cast<int32_t>(d1));
+        }
       }
       if (lane == 0) {
+        slot_of[warp] = slot;
         rng_lo[warp] = lo;
         rng_hi[warp] = hi;
       }
     }
     __syncthreads();
+    pending = false;
+    bool dirty = false;     // unsynchronised adds since the last barrier
     const int nt = min(kTermsPerPass, t1 - base);
     for (int w = 0; w < nt; ++w) {
-      for (int64_t p = rng_lo[w] + threadIdx.x; p < rng_hi[w]; p += blockDim.x)
-        acc[sp.post_doc[p] - d0] += sp.post_w[p];
-      __syncthreads();
+      const int slot = slot_of[w];
+      if (slot == kSkipTerm) continue;
+      if (slot >= 0) {
+        // Dense term: thread i owns float4 groups i, i + 256, ...; after
+        // another dense term nothing needs ordering.
+        if (pending) __syncthreads();
+        const float4* row = reinterpret_cast<const float4*>(sp.dense_w + slot * sp.dense_ld + d0);
+        for (int i = threadIdx.x; i < nv; i += blockDim.x) {
+          const float4 x = __ldg(row + i);
+          float4 a = acc4[i];
+          a.x += x.x;
+          a.y += x.y;
+          a.z += x.z;
+          a.w += x.w;
+          acc4[i] = a;
+        }
+        pending = false;
+        dirty = true;
+      } else {
+        if (dirty) __syncthreads();
+        const int64_t lo = rng_lo[w], hi = rng_hi[w];
+        for (int64_t p = lo + threadIdx.x; p < hi; p += kScatterUnroll * blockDim.x) {
+          int2 e[kScatterUnroll];
+#pragma unroll
+          for (int u = 0; u < kScatterUnroll; ++u) {
+            const int64_t pp = p + static_cast<int64_t>(u) * blockDim.x;
+            e[u] = pp < hi ? __ldg(sp.post + pp) : make_int2(-1, 0);
+          }
+#pragma unroll
+          for (int u = 0; u < kScatterUnroll; ++u)
+            if (e[u].x >= 0) acc[e[u].x - d0] += __int_as_float(e[u].y);
+        }
+        pending = true;
+        dirty = true;
+      }
     }
+    __syncthreads();        // the next pass rewrites the term table; the output reads acc
   }
 
   float m = 0.f;
-  float* orow = out + static_cast<int64_t>(qi) * ld;
-  for (int64_t dd = d0 + threadIdx.x; dd < d1; dd += blockDim.x) {
-    const float v = acc[dd - d0];
-    orow[dd] = v;
-    m = fmaxf(m, v);
+  float4* orow = reinterpret_cast<float4*>(out + static_cast<int64_t>(qi) * ld + d0);
+  for (int i = threadIdx.x; i < nv; i += blockDim.x) {
+    const float4 v = acc4[i];
+    orow[i] = v;
+    m = fmaxf(fmaxf(m, fmaxf(v.x, v.y)), fmaxf(v.z, v.w));
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));

@@ -98,12 +98,18 @@ cudaError_t launch_merge(const ListSet& ls, int q, int k, int64_t* out_ids, floa
                          cudaStream_t st, float* kth_out = nullptr);
 
 // --- BM25 matrix pass (lexical part of the hybrid search).
+// Per-posting weight w(t, d) = idf * tf (k1+1) / (tf + k1 (1 - b + b |d| / avgdl)).
+// Terms held by more than half of the chunks are stored as dense rows of
+// w(t, .) (zero where absent: 4 bytes per chunk instead of 8 per posting, and
+// no scatter); the other terms as postings.
 struct SparseIndex {
   int vocab;
-  int64_t nnz;               // postings
-  const int64_t* post_ptr;   // device, vocab + 1
-  const int32_t* post_doc;   // device, nnz, ascending per term
-  const float* post_w;       // device, nnz: idf * tf (k1+1) / (tf + k1 (1 - b + b |d| / avgdl))
+  int64_t nnz;               // postings of the sparse terms
+  const int64_t* post_ptr;   // device, vocab + 1 (empty range for dense terms)
+  const int2* post;          // device, nnz (chunk, weight bits), chunks ascending per term
+  const int32_t* dense_slot; // device, vocab: row of a dense term, -1 otherwise
+  const float* dense_w;      // device, rows x dense_ld
+  int64_t dense_ld;          // multiple of 4, >= n; zero past n
 };
 cudaError_t launch_bm25_matrix(const SparseIndex& sp, int64_t n, const int32_t* q_indptr,
                                const int32_t* q_terms, int q, float* out, int64_t ld,

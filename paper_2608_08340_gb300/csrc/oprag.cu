@@ -83,8 +83,10 @@ struct oprag_index {
   int vocab = 0;
   int64_t nnz = 0;
   int64_t* post_ptr = nullptr;
-  int32_t* post_doc = nullptr;
-  float* post_w = nullptr;
+  int2* post = nullptr;
+  int32_t* dense_slot = nullptr;
+  float* dense_w = nullptr;
+  int64_t dense_ld = 0;
 
   int opt_path = 0;
   int opt_block_n = 0;
@@ -129,11 +131,13 @@ struct oprag_index {
 
   void free_sparse() {
     if (post_ptr) cudaFree(post_ptr);
-    if (post_doc) cudaFree(post_doc);
-    if (post_w) cudaFree(post_w);
+    if (post) cudaFree(post);
+    if (dense_slot) cudaFree(dense_slot);
+    if (dense_w) cudaFree(dense_w);
     post_ptr = nullptr;
-    post_doc = nullptr;
-    post_w = nullptr;
+    post = nullptr;
+    dense_slot = nullptr;
+    dense_w = nullptr;
     has_sparse = false;
   }
 };
@@ -585,12 +589,18 @@ int oprag_index_set_sparse(oprag_index* idx, const int32_t* doc_indptr, const in
     }
   }
   const double avgdl = static_cast<double>(total) / static_cast<double>(n);
-  // Postings grouped by term, chunks ascending inside a term.
+  // Terms in more than half of the chunks become dense rows; the others
+  // keep postings grouped by term, chunks ascending inside a term.
+  std::vector<int32_t> slot(vocab, -1);
+  int n_dense = 0;
+  for (int t = 0; t < vocab; ++t)
+    if (2 * df[t] > n) slot[t] = n_dense++;
+  const int64_t dld = (n + 3) / 4 * 4;
+  std::vector<float> dense(static_cast<size_t>(n_dense) * dld, 0.f);
   std::vector<int64_t> ptr(static_cast<size_t>(vocab) + 1, 0);
-  for (int t = 0; t < vocab; ++t) ptr[t + 1] = ptr[t] + df[t];
+  for (int t = 0; t < vocab; ++t) ptr[t + 1] = ptr[t] + (slot[t] < 0 ? df[t] : 0);
   const int64_t nnz = ptr[vocab];
-  std::vector<int32_t> pdoc(nnz);
-  std::vector<float> pw(nnz);
+  std::vector<int2> post(nnz);
   std::vector<int64_t> fill(ptr.begin(), ptr.end() - 1);
   const double N = static_cast<double>(n);
   for (size_t i = 0; i < pair_doc.size(); ++i) {
@@ -600,9 +610,14 @@ int oprag_index_set_sparse(oprag_index* idx, const int32_t* doc_indptr, const in
     const double dft = static_cast<double>(df[t]);
     const double idf = std::log(1.0 + (N - dft + 0.5) / (dft + 0.5));
     const double tf = static_cast<double>(pair_tf[i]);
-    const int64_t at = fill[t]++;
-    pdoc[at] = dd;
-    pw[at] = static_cast<float>(idf * tf * (k1 + 1.0) / (tf + k1 * norm));
+    const float wt = static_cast<float>(idf * tf * (k1 + 1.0) / (tf + k1 * norm));
+    if (slot[t] >= 0) {
+      dense[static_cast<size_t>(slot[t]) * dld + dd] = wt;
+    } else {
+      int32_t bits;
+      std::memcpy(&bits, &wt, sizeof(bits));
+      post[fill[t]++] = make_int2(dd, bits);
+    }
   }
 
   DeviceGuard g(idx->device);
@@ -610,23 +625,27 @@ int oprag_index_set_sparse(oprag_index* idx, const int32_t* doc_indptr, const in
   if (e != cudaSuccess) return cuda_fail(e, "waiting for pending work");
   idx->free_sparse();
   if (cudaMalloc(&idx->post_ptr, ptr.size() * sizeof(int64_t)) != cudaSuccess ||
-      cudaMalloc(&idx->post_doc, std::max<int64_t>(nnz, 1) * sizeof(int32_t)) != cudaSuccess ||
-      cudaMalloc(&idx->post_w, std::max<int64_t>(nnz, 1) * sizeof(float)) != cudaSuccess) {
+      cudaMalloc(&idx->post, std::max<int64_t>(nnz, 1) * sizeof(int2)) != cudaSuccess ||
+      cudaMalloc(&idx->dense_slot, slot.size() * sizeof(int32_t)) != cudaSuccess ||
+      cudaMalloc(&idx->dense_w, std::max<size_t>(dense.size(), 4) * sizeof(float)) != cudaSuccess) {
     cudaGetLastError();
     idx->free_sparse();
     return fail(OPRAG_ERR_OOM, "cannot allocate postings");
   }
   e = cudaMemcpy(idx->post_ptr, ptr.data(), ptr.size() * sizeof(int64_t), cudaMemcpyHostToDevice);
   if (e == cudaSuccess && nnz)
-    e = cudaMemcpy(idx->post_doc, pdoc.data(), nnz * sizeof(int32_t), cudaMemcpyHostToDevice);
-  if (e == cudaSuccess && nnz)
-    e = cudaMemcpy(idx->post_w, pw.data(), nnz * sizeof(float), cudaMemcpyHostToDevice);
+    e = cudaMemcpy(idx->post, post.data(), nnz * sizeof(int2), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(idx->dense_slot, slot.data(), slot.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess && !dense.empty())
+    e = cudaMemcpy(idx->dense_w, dense.data(), dense.size() * sizeof(float), cudaMemcpyHostToDevice);
   if (e != cudaSuccess) {
     idx->free_sparse();
     return cuda_fail(e, "uploading postings");
   }
   idx->vocab = vocab;
   idx->nnz = nnz;
+  idx->dense_ld = dld;
   idx->has_sparse = true;
   return ok();
 }
@@ -648,7 +667,8 @@ int oprag_hybrid_search(oprag_index* idx, const void* queries, int32_t q, const 
                         sizeof(float) * static_cast<size_t>(qchunk * ld + qchunk), "BM25 block")))
     return rc;
   if ((rc = begin_call(idx, st))) return rc;
-  const SparseIndex sp{idx->vocab, idx->nnz, idx->post_ptr, idx->post_doc, idx->post_w};
+  const SparseIndex sp{idx->vocab,      idx->nnz,     idx->post_ptr, idx->post,
+                       idx->dense_slot, idx->dense_w, idx->dense_ld};
   const size_t qrow = static_cast<size_t>(idx->d) * elem_size(idx->dtype);
   for (int c0 = 0; c0 < q; c0 += qchunk) {
     const int qc = std::min(qchunk, q - c0);

@@ -1,6 +1,6 @@
 // Tensor-core search for bf16 indices on sm_103a: the query x chunk score
-// contraction of Sec. 4.4 ("dense scores ... vectorized matrix operations
-// over the embedding matrix") as a tcgen05 GEMM, with the partial top-k
+// contraction of Sec. 4.4 (dense scores of a query against the whole
+// embedding matrix in one matrix operation) as a tcgen05 GEMM, with the partial top-k
 // selection (Sec. 4.4, Sec. 7) fused into the epilogue so that the q x n
 // score matrix never reaches HBM.
 //
