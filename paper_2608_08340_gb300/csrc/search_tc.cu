@@ -114,14 +114,11 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
   if (!ok) per_tile = C;  // not expected; every slot then gets a list per tile
   pl.pmax = per_tile * epi_sets(list_len_for(s.k));
   const int K = list_len_for(s.k);
-  if (pair) {
-    pl.stages = stages_for<256, true>();
-    pl.smem = K <= 16 ? smem_for<256, 16, true>() : smem_for<256, 32, true>();
-  } else {
-    pl.stages = bn == 128 ? stages_for<128>() : stages_for<256>();
-    pl.smem = bn == 128 ? (K <= 16 ? smem_for<128, 16>() : smem_for<128, 32>())
-                        : (K <= 16 ? smem_for<256, 16>() : smem_for<256, 32>());
-  }
+  // Shared memory of the launch (the same sum as smem_for<BN, K, pair>).
+  const size_t b_stage = static_cast<size_t>(pair ? bn / 2 : bn) * 128;
+  pl.stages = pair ? stages_for<256, true>() : (bn == 128 ? stages_for<128>() : stages_for<256>());
+  pl.smem = static_cast<size_t>(pl.stages) * (kAStageBytes + b_stage) +
+            static_cast<size_t>(epi_sets(K)) * 128 * kStageRowBytes + 1024 + 256;
   return pl;
 }
 

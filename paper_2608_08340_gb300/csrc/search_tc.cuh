@@ -39,8 +39,10 @@ constexpr int kBlockM = 128;
 constexpr int kBlockK = 64;                 // bf16 per 128-byte row
 constexpr int kUmmaK = 16;
 // Epilogue warp sets: two (one per accumulator, 320 threads) for register
-// lists up to 16 keys; one set (192 threads, more registers per thread) for
-// the longer lists.
+// lists up to 16 keys; one set (192 threads) for the longer lists.  Ten warps
+// put three on two of the SM's four schedulers, which caps a thread at 168
+// registers; with six warps it may use 255 (measured: buffered lists with two
+// sets spill and run 11% slower).
 __host__ __device__ constexpr int epi_sets(int K) { return K <= 16 ? 2 : 1; }
 __host__ __device__ constexpr int threads_for(int K) { return 64 + 128 * epi_sets(K); }
 constexpr uint32_t kAStageBytes = kBlockM * kBlockK * 2;
