@@ -86,16 +86,28 @@ size_t tc_scratch_bytes(const SearchShape& s, const TcPlan& p);
 // qfloor (optional, q entries, register lists only): per-query k-th score
 // bounds shared by all lists, valid for entries tagged with gen (see
 // search_tc.cuh); zero-filled memory is a valid initial state.
+// levels / level_cnt (optional, q x kLevels, buffered lists only): candidate
+// floors and zeroed counters; a floor becomes a shared bound once k pushed
+// keys reach it.
 cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s, const Fusion& fu,
                              const TcPlan& plan, void* scratch, int* dev_err, ListSet* lists,
                              cudaStream_t st, const float* init_floor = nullptr,
-                             uint64_t* qfloor = nullptr, uint32_t gen = 0);
+                             uint64_t* qfloor = nullptr, uint32_t gen = 0,
+                             const float* levels = nullptr, int* level_cnt = nullptr);
 
 // --- final merge of partial lists into the sorted top-k per query.
 // kth_out (optional, q floats): the k-th best merged score of every query
-// (-inf when fewer than k candidates exist).
+// (-inf when fewer than k candidates exist).  levels_out (optional, q x
+// kLevels floats): the merged scores at ranks level_rank(k, i).
+constexpr int kLevels = 4;
+// Ranks k/16, k/8, k/4, k/2 (at least 1): candidate floors for a search of
+// k > 32 that a first pass over every 16th corpus tile proposes.
+inline __host__ __device__ int level_rank(int k, int i) {
+  const int r = k >> (kLevels - i);
+  return r < 1 ? 1 : r;
+}
 cudaError_t launch_merge(const ListSet& ls, int q, int k, int64_t* out_ids, float* out_scores,
-                         cudaStream_t st, float* kth_out = nullptr);
+                         cudaStream_t st, float* kth_out = nullptr, float* levels_out = nullptr);
 
 // --- BM25 matrix pass (lexical part of the hybrid search).
 // Per-posting weight w(t, d) = idf * tf (k1+1) / (tf + k1 (1 - b + b |d| / avgdl)).

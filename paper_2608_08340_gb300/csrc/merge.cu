@@ -34,7 +34,8 @@ __device__ __forceinline__ void offer32(WarpMerger<KP>& m, uint64_t key) {
 template <int KP>
 __global__ void __launch_bounds__(kMergeWarps * 32)
 merge_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
-             float* __restrict__ out_scores, float* __restrict__ kth_out) {
+             float* __restrict__ out_scores, float* __restrict__ kth_out,
+             float* __restrict__ levels_out) {
   constexpr int kCap = 2 * KP;
   extern __shared__ __align__(16) uint64_t smem_keys[];
   // Launched as a programmatic dependent of the search kernel: wait until
@@ -99,6 +100,10 @@ merge_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
     const uint64_t kk = f.sbuf[k - 1];
     kth_out[qi] = kk == kEmptyKey ? -INFINITY : key_score(kk);
   }
+  if (levels_out != nullptr && lane < kLevels) {
+    const uint64_t kk = f.sbuf[level_rank(k, lane) - 1];
+    levels_out[static_cast<int64_t>(qi) * kLevels + lane] = kk == kEmptyKey ? -INFINITY : key_score(kk);
+  }
   for (int i = lane; i < k; i += 32) {
     const uint64_t key = f.sbuf[i];
     const int64_t o = static_cast<int64_t>(qi) * k + i;
@@ -109,7 +114,7 @@ merge_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
 
 template <int KP>
 cudaError_t launch_merge_kp(const ListSet& ls, int q, int k, int64_t* ids, float* scores,
-                            cudaStream_t st, float* kth_out) {
+                            cudaStream_t st, float* kth_out, float* levels_out) {
   const size_t smem = static_cast<size_t>(kMergeWarps + 1) * 2 * KP * sizeof(uint64_t);
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(q);
@@ -121,7 +126,7 @@ cudaError_t launch_merge_kp(const ListSet& ls, int q, int k, int64_t* ids, float
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, merge_kernel<KP>, ls, q, k, ids, scores, kth_out);
+  return cudaLaunchKernelEx(&cfg, merge_kernel<KP>, ls, q, k, ids, scores, kth_out, levels_out);
 }
 
 // Few lists per query (at most 32): one warp per query merges the sorted
@@ -133,7 +138,8 @@ constexpr int kWayWarps = 8;        // queries per CTA
 
 __global__ void __launch_bounds__(kWayWarps * 32)
 merge_kway_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
-                  float* __restrict__ out_scores, float* __restrict__ kth_out) {
+                  float* __restrict__ out_scores, float* __restrict__ kth_out,
+                  float* __restrict__ levels_out) {
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int qi = blockIdx.x * kWayWarps + warp;
@@ -187,13 +193,16 @@ merge_kway_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
     }
     if (r == k - 1 && kth_out != nullptr && lane == 0)
       kth_out[qi] = best == kEmptyKey ? -INFINITY : key_score(best);
+    if (levels_out != nullptr && lane < kLevels && r == level_rank(k, lane) - 1)
+      levels_out[static_cast<int64_t>(qi) * kLevels + lane] =
+          best == kEmptyKey ? -INFINITY : key_score(best);
   }
 }
 
 }  // namespace
 
 cudaError_t launch_merge(const ListSet& ls, int q, int k, int64_t* out_ids, float* out_scores,
-                         cudaStream_t st, float* kth_out) {
+                         cudaStream_t st, float* kth_out, float* levels_out) {
   if (q <= 0) return cudaSuccess;
   if (ls.P <= 32) {
     cudaLaunchConfig_t cfg{};
@@ -206,12 +215,13 @@ cudaError_t launch_merge(const ListSet& ls, int q, int k, int64_t* out_ids, floa
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, merge_kway_kernel, ls, q, k, out_ids, out_scores, kth_out);
+    return cudaLaunchKernelEx(&cfg, merge_kway_kernel, ls, q, k, out_ids, out_scores, kth_out,
+                              levels_out);
   }
-  if (k <= 32) return launch_merge_kp<32>(ls, q, k, out_ids, out_scores, st, kth_out);
-  if (k <= 64) return launch_merge_kp<64>(ls, q, k, out_ids, out_scores, st, kth_out);
-  if (k <= 128) return launch_merge_kp<128>(ls, q, k, out_ids, out_scores, st, kth_out);
-  return launch_merge_kp<256>(ls, q, k, out_ids, out_scores, st, kth_out);
+  if (k <= 32) return launch_merge_kp<32>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
+  if (k <= 64) return launch_merge_kp<64>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
+  if (k <= 128) return launch_merge_kp<128>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
+  return launch_merge_kp<256>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
 }
 
 }  // namespace oprag

@@ -236,17 +236,22 @@ int run_search(oprag_index* idx, const void* Q, int q, int k, const Fusion& fu, 
     s32.k = 32;
     TcPlan splan{};
     size_t sample_bytes = 0;
+    // Sampled-pass scratch: its lists, its merged top-k (ids + scores), then
+    // per query the k-th score, kLevels counted floors and their counters.
+    const size_t per_query_tail = sizeof(float) + kLevels * (sizeof(float) + sizeof(int));
     if (sampled) {
       splan = tc_plan(s32, idx->num_sms, plan.block_n, kSampleStride, plan.pair, pair_capacity(idx));
       sample_bytes = (tc_scratch_bytes(s32, splan) + 255) / 256 * 256 +
                      (static_cast<size_t>(q) * k * 12 + 255) / 256 * 256 +
-                     static_cast<size_t>(q) * sizeof(float);
+                     static_cast<size_t>(q) * per_query_tail + 16;
     }
     int rc = idx->ensure(&idx->scratch, &idx->scratch_bytes, main_bytes + sample_bytes,
                          "search scratch");
     if (rc) return rc;
     if (idx->timing) cudaEventRecord(idx->ev[1], st);
     const float* floor = nullptr;
+    float* levels = nullptr;
+    int* level_cnt = nullptr;
     if (sampled) {
       char* sbase = static_cast<char*>(idx->scratch) + main_bytes;
       const size_t slist = (tc_scratch_bytes(s32, splan) + 255) / 256 * 256;
@@ -254,9 +259,14 @@ int run_search(oprag_index* idx, const void* Q, int q, int k, const Fusion& fu, 
       float* sscores = reinterpret_cast<float*>(sids + static_cast<size_t>(q) * k);
       float* kth = reinterpret_cast<float*>(
           sbase + slist + (static_cast<size_t>(q) * k * 12 + 255) / 256 * 256);
+      // 16-byte aligned: each query's kLevels counters are read as one int4.
+      levels = kth + (static_cast<size_t>(q) + 3) / 4 * 4;
+      level_cnt = reinterpret_cast<int*>(levels + static_cast<size_t>(q) * kLevels);
       ListSet slists{};
       e = launch_tc_search(idx->emb, Q, s32, fu, splan, sbase, idx->dev_err, &slists, st);
-      if (e == cudaSuccess) e = launch_merge(slists, q, k, sids, sscores, st, kth);
+      if (e == cudaSuccess) e = launch_merge(slists, q, k, sids, sscores, st, kth, levels);
+      if (e == cudaSuccess)
+        e = cudaMemsetAsync(level_cnt, 0, static_cast<size_t>(q) * kLevels * sizeof(int), st);
       if (e != cudaSuccess) return cuda_fail(e, "sampling pass");
       floor = kth;
     }
@@ -266,7 +276,7 @@ int run_search(oprag_index* idx, const void* Q, int q, int k, const Fusion& fu, 
       if ((rc = shared_floors(idx, q, st, &qf, &gen))) return rc;
     }
     e = launch_tc_search(idx->emb, Q, s, fu, plan, idx->scratch, idx->dev_err, &lists, st, floor,
-                         qf, gen);
+                         qf, gen, levels, level_cnt);
     plan_used = plan;
   }
   if (e != cudaSuccess) return cuda_fail(e, "search kernel");

@@ -140,7 +140,7 @@ size_t tc_scratch_bytes(const SearchShape& s, const TcPlan& pl) {
 cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s, const Fusion& fu,
                              const TcPlan& pl, void* scratch, int* dev_err, ListSet* lists,
                              cudaStream_t st, const float* init_floor, uint64_t* qfloor,
-                             uint32_t gen) {
+                             uint32_t gen, const float* levels, int* level_cnt) {
   CUtensorMap mq, me;
   // With a single query tile only its real rows are loaded (the remaining
   // rows of the A tile hold stale data whose TMEM lanes the epilogue never
@@ -172,8 +172,11 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
   prm.meta_worst = prm.lists + rows * stride;
   prm.meta_count = reinterpret_cast<int*>(prm.meta_worst + (K > 32 ? rows : 0));
   prm.dev_err = dev_err;
+  // Register lists publish their k-th scores; buffered lists use counted floors.
   prm.qfloor = K <= 32 ? qfloor : nullptr;
   prm.gen = gen;
+  prm.levels = K > 32 ? levels : nullptr;
+  prm.level_cnt = K > 32 ? level_cnt : nullptr;
   lists->keys = prm.lists;
   lists->P = pl.pmax;
   lists->TH = kBlockM;

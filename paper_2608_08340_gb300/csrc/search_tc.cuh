@@ -71,6 +71,11 @@ struct TcParams {
   // other searches read as -inf); see shared_floor_read.
   uint64_t* qfloor;
   uint32_t gen;
+  // Optional (buffered lists): per query, kLevels candidate floors (best
+  // first) and counters of pushed keys reaching each; a floor whose counter
+  // reached k bounds the query's k-th best score for every list.
+  const float* levels;
+  int* level_cnt;
 };
 
 // Units of one CTA in processing order.  The corpus tiles are cut into
@@ -448,6 +453,24 @@ template <int K>
 struct EpiList<K, true> {
   static constexpr int kStride = 2 * K;
   BufTopK<K> t;
+  // Counted floors of the current query (see TcParams::levels).
+  float lvl[kLevels];
+  int* cnt;
+  __device__ __forceinline__ void set_query(const TcParams& p, int64_t q_index, bool valid) {
+    cnt = valid && p.levels != nullptr ? p.level_cnt + q_index * kLevels : nullptr;
+#pragma unroll
+    for (int i = 0; i < kLevels; ++i) lvl[i] = cnt != nullptr ? p.levels[q_index * kLevels + i] : INFINITY;
+  }
+  // The best counted floor that k pushed keys already reach (-inf if none).
+  __device__ __forceinline__ float proven_floor(int k) const {
+    if (cnt == nullptr) return -INFINITY;
+    const int4 c = __ldcg(reinterpret_cast<const int4*>(cnt));
+    const int cs[kLevels] = {c.x, c.y, c.z, c.w};
+    float f = -INFINITY;
+#pragma unroll
+    for (int i = kLevels - 1; i >= 0; --i) f = cs[i] >= k ? lvl[i] : f;
+    return f;
+  }
   __device__ __forceinline__ void init_mem(const TcParams& p, int64_t sr, int qidx) {
     p.meta_count[sr] = 0;
     // A known lower bound f of the k-th best score admits only scores >= f
@@ -470,12 +493,26 @@ struct EpiList<K, true> {
     t.count = 0;
     t.worst = kEmptyKey;
     t.floor = -INFINITY;
+    cnt = nullptr;
   }
   __device__ __forceinline__ bool full() const { return t.worst != kEmptyKey; }
   __device__ __forceinline__ float floor() const { return t.floor; }
   __device__ __forceinline__ void push(float s, uint32_t id) { t.push(s, id); }
+  // Pushes a candidate; a pushed key that reaches a counted floor counts
+  // towards it (fire-and-forget adds).  k counts prove k real keys >= that
+  // floor, which then bounds the query's k-th best for every list; a pushed
+  // key leaves its list only when the list holds K >= k better keys, so the
+  // proof stays valid.
   __device__ __forceinline__ void insert(float s, uint32_t id) {
-    if (s > -INFINITY) t.push(s, id);
+    if (!(s > -INFINITY)) return;
+    const uint64_t key = make_key(s, id);
+    if (key <= t.worst) return;
+    t.buf[t.count++] = key;
+    if (cnt != nullptr) {
+#pragma unroll
+      for (int i = 0; i < kLevels; ++i)
+        if (s >= lvl[i]) atomicAdd(cnt + i, 1);
+    }
   }
   __device__ __forceinline__ void sync(bool final, bool active) { t.sync(final, active); }
   // Warp-collective: sorts the lane's buffer, best K first.
@@ -710,12 +747,17 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         cur_sr = list_row(J);
         cur_valid = valid && owns(J);
         if (cur_valid) list.load(p, cur_sr); else list.clear();
+        if constexpr (K > 32) list.set_query(p, static_cast<int64_t>(j) * kBlockM + row, cur_valid);
       }
       const bool act = cur_valid;
       // Shared bound of this query's k-th best score, read while the MMAs run.
       float gfl = -INFINITY;
-      if (K <= 32 && p.qfloor != nullptr && act)
-        gfl = shared_floor_read(p.qfloor, static_cast<int64_t>(j) * kBlockM + row, p.gen);
+      if constexpr (K <= 32) {
+        if (p.qfloor != nullptr && act)
+          gfl = shared_floor_read(p.qfloor, static_cast<int64_t>(j) * kBlockM + row, p.gen);
+      } else {
+        if (act) gfl = list.proven_floor(p.k);
+      }
       if (!mbar_wait(&tfull[acc], (acc_ph >> acc) & 1u, abort_flag, p.dev_err)) break;
       tc_fence_after();
       if (warp_live) {
@@ -773,8 +815,11 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             // so the warp runs max-per-lane rounds instead of the sum.
             uint32_t mask = 0;
             if (act) {
+              // Four independent 8-bit parts (short dependency chains).
+              uint32_t part[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
-              for (int i = 0; i < 32; ++i) mask |= (v[i] >= fl ? 1u : 0u) << i;
+              for (int i = 0; i < 32; ++i) part[i >> 3] |= (v[i] >= fl ? 1u : 0u) << i;
+              mask = (part[0] | part[1]) | (part[2] | part[3]);
 #pragma unroll
               for (int g = 0; g < 8; ++g)
                 *reinterpret_cast<float4*>(srow + ((g ^ swz) << 2)) =
