@@ -183,6 +183,12 @@ OPRAG_API int oprag_index_set_option(oprag_index *idx, int32_t option, int32_t v
  * every CTA on its own (M = 128 MMAs). */
 #define OPRAG_OPT_PAIR 4
 
+/* OPRAG_OPT_BOUND_TAG (test hook): sets the 32-bit tag of the last search's
+ * shared k-th score bounds (bit pattern of value); the next searches use the
+ * following tags, so a test can make them wrap around (the bounds array is
+ * then cleared). */
+#define OPRAG_OPT_BOUND_TAG 5
+
 /* OPRAG_OPT_TIMING: 1 makes every later search record CUDA events, on the
  * call's stream, around its lexical (BM25) kernel, its main search kernel and
  * its merge kernel; oprag_index_last_timing() reads them.  0 (default) off. */

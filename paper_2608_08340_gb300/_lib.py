@@ -16,6 +16,7 @@ OPRAG_OPT_PATH = 1
 OPRAG_OPT_BLOCK_N = 2
 OPRAG_OPT_TIMING = 3
 OPRAG_OPT_PAIR = 4
+OPRAG_OPT_BOUND_TAG = 5
 
 ERRORS = {
     0: "OK",

@@ -1,115 +1,32 @@
 // Global top-k reduction: merges the partial lists that the search kernels
 // leave per (query tile, producer) into the final ranked top-k of each query.
-// This is the "local candidates, then global top-k reduction" step of
-// Op_retrieve (Sec. 3.2; Sec. 4.1 Retrieval), done inside one GPU: the
-// producers are corpus slices instead of index shards.
+// This is the step of Op_retrieve (Sec. 3.2; Sec. 4.1 Retrieval) that reduces
+// local candidates to the global top-k, done inside one GPU: the producers
+// are corpus slices instead of index shards.
 //
-// Many lists (more than 32 per query): one CTA per query.  The P * k
-// candidate keys of a query (the first k of each
-// producer's sorted list) are split evenly over the warps; a warp fetches four
-// 32-key groups at once (independent loads, so L2 latency is paid once per
-// group of four, not once per list) and filters them against its running
-// k-th best.  Warp 0 then merges the warps' results.
-#include "common.cuh"
-#include "internal.h"
+// Many lists (more than 32 per query): one CTA per query runs the block merge
+// of merge.cuh.
+#include "merge.cuh"
 
 namespace oprag {
 
 namespace {
 
 constexpr int kMergeWarps = 8;
-constexpr int kUnroll = 4;
-
-template <int KP>
-__device__ __forceinline__ void offer32(WarpMerger<KP>& m, uint64_t key) {
-  const int lane = threadIdx.x & 31;
-  const bool pass = key > m.worst;
-  const uint32_t bits = __ballot_sync(0xffffffffu, pass);
-  if (bits == 0) return;
-  if (m.count > WarpMerger<KP>::kCap - 32) m.compact();
-  if (pass) m.sbuf[m.count + __popc(bits & ((1u << lane) - 1u))] = key;
-  m.count += __popc(bits);
-}
 
 template <int KP>
 __global__ void __launch_bounds__(kMergeWarps * 32)
 merge_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
              float* __restrict__ out_scores, float* __restrict__ kth_out,
              float* __restrict__ levels_out) {
-  constexpr int kCap = 2 * KP;
   extern __shared__ __align__(16) uint64_t smem_keys[];
   // Launched as a programmatic dependent of the search kernel: wait until
   // that grid has finished and its lists are visible.
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int qi = blockIdx.x;
   if (qi >= q) return;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int tile = qi / ls.TH, row = qi % ls.TH;
-  const uint64_t* base = ls.keys + (static_cast<int64_t>(tile) * ls.P * ls.TH + row) * ls.stride;
-  const int64_t list_step = static_cast<int64_t>(ls.TH) * ls.stride;
-  int np = ls.P;
-  if (ls.C > 0) {
-    int c0 = static_cast<int>(static_cast<int64_t>(tile / ls.pair) * ls.C / ls.qt) - 1;
-    c0 = c0 < 0 ? 0 : c0;
-    np = min(ls.P, (ls.C - c0) * ls.sets);
-  }
-  const int kl = min(k, ls.klen);         // keys read from each list
-  const int total = np * kl;
-  const int lo = static_cast<int>(static_cast<int64_t>(total) * warp / kMergeWarps);
-  const int hi = static_cast<int>(static_cast<int64_t>(total) * (warp + 1) / kMergeWarps);
-
-  WarpMerger<KP> m;
-  m.init(smem_keys + warp * kCap, k);
-  for (int g = lo; g < hi; g += 32 * kUnroll) {
-    uint64_t key[kUnroll];
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int i = g + u * 32 + lane;
-      key[u] = kEmptyKey;
-      if (i < hi) {
-        const int p = i / kl;
-        key[u] = base[p * list_step + (i - p * kl)];
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) offer32(m, key[u]);
-  }
-  m.finish();
-  __syncthreads();
-  if (warp != 0) return;
-
-  WarpMerger<KP> f;
-  f.init(smem_keys + kMergeWarps * kCap, k);
-  const int all = kMergeWarps * k;
-  for (int g = 0; g < all; g += 32 * kUnroll) {
-    uint64_t key[kUnroll];
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int i = g + u * 32 + lane;
-      key[u] = kEmptyKey;
-      if (i < all) {
-        const int w = i / k;
-        key[u] = smem_keys[w * kCap + (i - w * k)];
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) offer32(f, key[u]);
-  }
-  f.finish();
-  if (kth_out != nullptr && lane == 0) {
-    const uint64_t kk = f.sbuf[k - 1];
-    kth_out[qi] = kk == kEmptyKey ? -INFINITY : key_score(kk);
-  }
-  if (levels_out != nullptr && lane < kLevels) {
-    const uint64_t kk = f.sbuf[level_rank(k, lane) - 1];
-    levels_out[static_cast<int64_t>(qi) * kLevels + lane] = kk == kEmptyKey ? -INFINITY : key_score(kk);
-  }
-  for (int i = lane; i < k; i += 32) {
-    const uint64_t key = f.sbuf[i];
-    const int64_t o = static_cast<int64_t>(qi) * k + i;
-    out_ids[o] = key == kEmptyKey ? -1 : static_cast<int64_t>(key_id(key));
-    out_scores[o] = key == kEmptyKey ? -INFINITY : key_score(key);
-  }
+  merge_one_query<KP, false>(ls, qi, k, kMergeWarps, out_ids, out_scores, kth_out, levels_out,
+                             smem_keys);
 }
 
 template <int KP>
@@ -145,12 +62,7 @@ merge_kway_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
   const int qi = blockIdx.x * kWayWarps + warp;
   if (qi >= q) return;
   const int tile = qi / ls.TH, row = qi % ls.TH;
-  int np = ls.P;
-  if (ls.C > 0) {
-    int c0 = static_cast<int>(static_cast<int64_t>(tile / ls.pair) * ls.C / ls.qt) - 1;
-    c0 = c0 < 0 ? 0 : c0;
-    np = min(ls.P, (ls.C - c0) * ls.sets);
-  }
+  const int np = merge_list_count(ls, tile);
   const int kl = min(k, ls.klen);
   const uint64_t* list = ls.keys + ((static_cast<int64_t>(tile) * ls.P + lane) * ls.TH + row) *
                                        static_cast<int64_t>(ls.stride);

@@ -732,6 +732,10 @@ int oprag_index_set_option(oprag_index* idx, int32_t option, int32_t value) {
     idx->timing = value != 0;
     return ok();
   }
+  if (option == OPRAG_OPT_BOUND_TAG) {
+    idx->gen = static_cast<uint32_t>(value);
+    return ok();
+  }
   if (option == OPRAG_OPT_PAIR) {
     if (value < 0 || value > 2) return fail(OPRAG_ERR_INVALID_ARG, "pair mode %d", value);
     idx->opt_pair = value;

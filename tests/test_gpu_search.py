@@ -216,3 +216,25 @@ def test_large_k_with_sampled_floor(k):
     rows = np.sort(rng.choice(q, 12, replace=False))
     check_dense(ids, sc, E, Q, k, f"large k={k}", rows=rows)
     idx.check()
+
+
+def test_shared_bound_tags_wrap_around():
+    """Searches share per-query k-th score bounds tagged with a 32-bit
+    generation; when the tag wraps, the bounds array is cleared.  Results
+    across the wrap must equal those of a fresh index."""
+    from paper_2608_08340_gb300 import _lib
+    w = workloads.config(1, n=20000, batch=300)
+    ref = _index(w.E_data)
+    r_ids, r_sc = ref.search(dev_tensor(w.Q_data), 10)
+    idx = _index(w.E_data)
+    # Corpus rows as queries: their bounds (self-matches, scores near 1) would
+    # wreck the next queries' results if an entry of this search were ever
+    # read as current.  This search gets tag 1; the wrap below reuses tag 1.
+    idx.search(dev_tensor(w.E_data[:300]), 10)
+    idx.set_option(_lib.OPRAG_OPT_BOUND_TAG, -3)         # tag 0xFFFFFFFD
+    for _ in range(4):                                   # 0xFFFFFFFE, 0xFFFFFFFF, wrap to 1, 2
+        ids, sc = idx.search(dev_tensor(w.Q_data), 10)
+        torch.cuda.synchronize()
+        assert torch.equal(ids, r_ids)
+        assert (sc - r_sc).abs().max().item() == 0.0
+    idx.check()
