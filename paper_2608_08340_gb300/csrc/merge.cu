@@ -111,25 +111,103 @@ merge_kway_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
   }
 }
 
+// Between 33 and 64 lists and k <= 16: one warp per query.  Lane l keeps, sorted in registers, the
+// best KL keys among the lists l, l + 32, ... (each list's kl keys are
+// contiguous and sorted; all loads of a lane are independent); then the
+// lanes' sorted lists are merged head by head as above.
+template <int KL>
+__global__ void __launch_bounds__(kWayWarps * 32)
+merge_small_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
+                   float* __restrict__ out_scores, float* __restrict__ kth_out,
+                   float* __restrict__ levels_out) {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qi = blockIdx.x * kWayWarps + warp;
+  if (qi >= q) return;
+  const int tile = qi / ls.TH, row = qi % ls.TH;
+  const int np = merge_list_count(ls, tile);
+  const int kl = min(k, ls.klen);
+  const uint64_t* base = ls.keys + (static_cast<int64_t>(tile) * ls.P * ls.TH + row) * ls.stride;
+  const int64_t list_step = static_cast<int64_t>(ls.TH) * ls.stride;
+  uint64_t top[KL];
+#pragma unroll
+  for (int i = 0; i < KL; ++i) top[i] = kEmptyKey;
+  for (int pl = lane; pl < np; pl += 32) {
+    const uint64_t* list = base + pl * list_step;
+    uint64_t key[KL];
+#pragma unroll
+    for (int i = 0; i < KL; ++i) key[i] = i < kl ? list[i] : kEmptyKey;
+#pragma unroll
+    for (int j = 0; j < KL; ++j) {
+      const uint64_t x = key[j];
+      if (x > top[KL - 1]) {
+#pragma unroll
+        for (int i = KL - 1; i > 0; --i)
+          top[i] = x > top[i - 1] ? top[i - 1] : (x > top[i] ? x : top[i]);
+        top[0] = x > top[0] ? x : top[0];
+      }
+    }
+  }
+  uint64_t mine = kEmptyKey;
+  for (int r = 0; r < k; ++r) {
+    uint64_t best = top[0];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) best = umax64(best, __shfl_xor_sync(0xffffffffu, best, o));
+    if (best != kEmptyKey && top[0] == best) {
+#pragma unroll
+      for (int i = 0; i + 1 < KL; ++i) top[i] = top[i + 1];
+      top[KL - 1] = kEmptyKey;
+    }
+    if ((r & 31) == lane) mine = best;
+    if ((r & 31) == 31 || r == k - 1) {
+      const int i = (r & ~31) + lane;
+      if (i <= r) {
+        const int64_t o = static_cast<int64_t>(qi) * k + i;
+        out_ids[o] = mine == kEmptyKey ? -1 : static_cast<int64_t>(key_id(mine));
+        out_scores[o] = mine == kEmptyKey ? -INFINITY : key_score(mine);
+      }
+    }
+    if (r == k - 1 && kth_out != nullptr && lane == 0)
+      kth_out[qi] = best == kEmptyKey ? -INFINITY : key_score(best);
+    if (levels_out != nullptr && lane < kLevels && r == level_rank(k, lane) - 1)
+      levels_out[static_cast<int64_t>(qi) * kLevels + lane] =
+          best == kEmptyKey ? -INFINITY : key_score(best);
+  }
+}
+
+template <typename Kern>
+cudaError_t launch_warp_per_query(Kern kern, const ListSet& ls, int q, int k, int64_t* out_ids,
+                                  float* out_scores, cudaStream_t st, float* kth_out,
+                                  float* levels_out) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((q + kWayWarps - 1) / kWayWarps);
+  cfg.blockDim = dim3(kWayWarps * 32);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, ls, q, k, out_ids, out_scores, kth_out, levels_out);
+}
+
 }  // namespace
 
 cudaError_t launch_merge(const ListSet& ls, int q, int k, int64_t* out_ids, float* out_scores,
                          cudaStream_t st, float* kth_out, float* levels_out) {
   if (q <= 0) return cudaSuccess;
-  if (ls.P <= 32) {
-    cudaLaunchConfig_t cfg{};
-    cfg.gridDim = dim3((q + kWayWarps - 1) / kWayWarps);
-    cfg.blockDim = dim3(kWayWarps * 32);
-    cfg.dynamicSmemBytes = 0;
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, merge_kway_kernel, ls, q, k, out_ids, out_scores, kth_out,
-                              levels_out);
-  }
+  if (ls.P <= 32)
+    return launch_warp_per_query(merge_kway_kernel, ls, q, k, out_ids, out_scores, st, kth_out,
+                                 levels_out);
+  // Up to 64 lists a lane walks at most two; with more, the block merge's
+  // eight warps per query keep the loads in flight (measured on GB300).
+  if (ls.P <= 64 && k <= 8)
+    return launch_warp_per_query(merge_small_kernel<8>, ls, q, k, out_ids, out_scores, st,
+                                 kth_out, levels_out);
+  if (ls.P <= 64 && k <= 16)
+    return launch_warp_per_query(merge_small_kernel<16>, ls, q, k, out_ids, out_scores, st,
+                                 kth_out, levels_out);
   if (k <= 32) return launch_merge_kp<32>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
   if (k <= 64) return launch_merge_kp<64>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
   if (k <= 128) return launch_merge_kp<128>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
