@@ -111,35 +111,49 @@ merge_kway_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
   }
 }
 
-// Between 33 and 64 lists and k <= 16: one warp per query.  Lane l keeps, sorted in registers, the
-// best KL keys among the lists l, l + 32, ... (each list's kl keys are
-// contiguous and sorted; all loads of a lane are independent); then the
-// lanes' sorted lists are merged head by head as above.
+// More than 32 lists and k <= 16: one warp per query, two queries per CTA of
+// 64 threads with at most 64 registers a thread, so that a CTA fits on an SM
+// beside a running search CTA: launched early (programmatic dependent launch),
+// it waits in place and starts as soon as the search grid ends.  Lane l reads
+// the keys l, l + 32, ... of the query's np * kl candidates (64 / KL
+// independent loads at a time, within the register budget) and keeps the
+// best KL sorted in registers;
+// then the lanes' sorted lists are merged head by head as above.
+constexpr int kSmallWarps = 2;
+
 template <int KL>
-__global__ void __launch_bounds__(kWayWarps * 32)
+__global__ void __launch_bounds__(kSmallWarps * 32, 16)
 merge_small_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
                    float* __restrict__ out_scores, float* __restrict__ kth_out,
                    float* __restrict__ levels_out) {
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int qi = blockIdx.x * kWayWarps + warp;
+  const int qi = blockIdx.x * kSmallWarps + warp;
   if (qi >= q) return;
   const int tile = qi / ls.TH, row = qi % ls.TH;
   const int np = merge_list_count(ls, tile);
   const int kl = min(k, ls.klen);
+  const int total = np * kl;
   const uint64_t* base = ls.keys + (static_cast<int64_t>(tile) * ls.P * ls.TH + row) * ls.stride;
   const int64_t list_step = static_cast<int64_t>(ls.TH) * ls.stride;
+  constexpr int kLoadBatch = 64 / KL;
   uint64_t top[KL];
 #pragma unroll
   for (int i = 0; i < KL; ++i) top[i] = kEmptyKey;
-  for (int pl = lane; pl < np; pl += 32) {
-    const uint64_t* list = base + pl * list_step;
-    uint64_t key[KL];
+  for (int g = lane; g < total; g += 32 * kLoadBatch) {
+    uint64_t key[kLoadBatch];
 #pragma unroll
-    for (int i = 0; i < KL; ++i) key[i] = i < kl ? list[i] : kEmptyKey;
+    for (int u = 0; u < kLoadBatch; ++u) {
+      const int i = g + 32 * u;
+      key[u] = kEmptyKey;
+      if (i < total) {
+        const int pl = i / kl;
+        key[u] = base[pl * list_step + (i - pl * kl)];
+      }
+    }
 #pragma unroll
-    for (int j = 0; j < KL; ++j) {
-      const uint64_t x = key[j];
+    for (int u = 0; u < kLoadBatch; ++u) {
+      const uint64_t x = key[u];
       if (x > top[KL - 1]) {
 #pragma unroll
         for (int i = KL - 1; i > 0; --i)
@@ -176,12 +190,12 @@ merge_small_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
 }
 
 template <typename Kern>
-cudaError_t launch_warp_per_query(Kern kern, const ListSet& ls, int q, int k, int64_t* out_ids,
-                                  float* out_scores, cudaStream_t st, float* kth_out,
-                                  float* levels_out) {
+cudaError_t launch_warp_per_query(Kern kern, int warps, const ListSet& ls, int q, int k,
+                                  int64_t* out_ids, float* out_scores, cudaStream_t st,
+                                  float* kth_out, float* levels_out) {
   cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3((q + kWayWarps - 1) / kWayWarps);
-  cfg.blockDim = dim3(kWayWarps * 32);
+  cfg.gridDim = dim3((q + warps - 1) / warps);
+  cfg.blockDim = dim3(warps * 32);
   cfg.dynamicSmemBytes = 0;
   cfg.stream = st;
   cudaLaunchAttribute attr[1];
@@ -198,16 +212,14 @@ cudaError_t launch_merge(const ListSet& ls, int q, int k, int64_t* out_ids, floa
                          cudaStream_t st, float* kth_out, float* levels_out) {
   if (q <= 0) return cudaSuccess;
   if (ls.P <= 32)
-    return launch_warp_per_query(merge_kway_kernel, ls, q, k, out_ids, out_scores, st, kth_out,
-                                 levels_out);
-  // Up to 64 lists a lane walks at most two; with more, the block merge's
-  // eight warps per query keep the loads in flight (measured on GB300).
-  if (ls.P <= 64 && k <= 8)
-    return launch_warp_per_query(merge_small_kernel<8>, ls, q, k, out_ids, out_scores, st,
+    return launch_warp_per_query(merge_kway_kernel, kWayWarps, ls, q, k, out_ids, out_scores, st,
                                  kth_out, levels_out);
-  if (ls.P <= 64 && k <= 16)
-    return launch_warp_per_query(merge_small_kernel<16>, ls, q, k, out_ids, out_scores, st,
-                                 kth_out, levels_out);
+  if (k <= 8)
+    return launch_warp_per_query(merge_small_kernel<8>, kSmallWarps, ls, q, k, out_ids,
+                                 out_scores, st, kth_out, levels_out);
+  if (k <= 16)
+    return launch_warp_per_query(merge_small_kernel<16>, kSmallWarps, ls, q, k, out_ids,
+                                 out_scores, st, kth_out, levels_out);
   if (k <= 32) return launch_merge_kp<32>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
   if (k <= 64) return launch_merge_kp<64>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
   if (k <= 128) return launch_merge_kp<128>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
