@@ -50,10 +50,12 @@ cudaError_t launch_merge_kp(const ListSet& ls, int q, int k, int64_t* ids, float
 // lists directly.  Lane l holds the head of list l (with the next keys
 // prefetched in registers); each round the warp takes the largest head
 // (keys are unique, so exactly one lane wins) and that lane advances.
-constexpr int kHeads = 16;          // keys prefetched per list
-constexpr int kWayWarps = 8;        // queries per CTA
+// CTAs of two warps under 64 registers a thread fit beside a running search
+// CTA, so the early-launched merge waits in place.
+constexpr int kHeads = 8;           // keys prefetched per list
+constexpr int kWayWarps = 2;        // queries per CTA
 
-__global__ void __launch_bounds__(kWayWarps * 32)
+__global__ void __launch_bounds__(kWayWarps * 32, 16)
 merge_kway_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
                   float* __restrict__ out_scores, float* __restrict__ kth_out,
                   float* __restrict__ levels_out) {
