@@ -29,10 +29,11 @@ def _noalloc(lib, idx, Q, k):
     return rc, ids, sc
 
 
-@pytest.mark.parametrize("cfg,q,k", [(1, 256, 5), (1, 1, 5), (2, 300, 10), (0, 16, 5)])
-def test_noalloc_matches_search_twice(cfg, q, k):
+@pytest.mark.parametrize("cfg,q,k,n", [(1, 256, 5, 20000), (1, 1, 5, 20000), (2, 300, 10, 20000),
+                                       (0, 16, 5, None), (1, 64, 100, 2000)])
+def test_noalloc_matches_search_twice(cfg, q, k, n):
     lib = _lib.load()
-    w = workloads.config(cfg, batch=q, n=20000 if cfg != 0 else None)
+    w = workloads.config(cfg, batch=q, n=n)
     idx = Index(dev_tensor(w.E_data))
     Q = dev_tensor(w.Q_data)
     ref_ids, ref_sc = idx.search(Q, k)
