@@ -25,6 +25,7 @@ import argparse
 import hashlib
 import json
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -39,64 +40,23 @@ sys.path.insert(0, ROOT)
 from paper_2608_08340_gb300 import workloads  # noqa: E402
 
 L2_FLUSH_BYTES = 512 << 20
-KERNEL_SOURCES = ["common.cuh", "search_tc.cuh", "search_tc.cu", "search_simt.cuh", "merge.cu",
-                  "bm25.cu", "upsert.cu"]
+# Files that define the search kernel whose DRAM traffic profiles/ncu_traffic.json
+# records; the hash covers their code with comments and blank space removed.
+KERNEL_SOURCES = ["common.cuh", "search_tc.cuh", "search_tc.cu"]
 
 
-def parse():
-    p = argparse.ArgumentParser()
-    p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=200)
-    p.add_argument("--warmup", type=int, default=10)
-    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    p.add_argument("--config", type=int, default=1)
-    p.add_argument("--batch", type=int, default=None)
-    p.add_argument("--no-cpu-baseline", action="store_true")
-    p.add_argument("--block-n", type=int, default=0, help="tensor-core tile rows (0 = auto)")
-    p.add_argument("--path", choices=["auto", "simt", "tc"], default="auto")
-    p.add_argument("--pair", choices=["auto", "single", "pair"], default="auto",
-                   help="tensor-core kernel: CTA pairs (M = 256 MMAs) or single CTAs")
-    return p.parse_args()
+def _code_only(text: str) -> str:
+    text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", " ", text)
+    return " ".join(text.split())
 
 
-def default_batch(cfg: int) -> int:
-    return {0: 16, 1: 256, 2: 4096, 3: 1024, 4: 2048}[cfg]
-
-
-def workload_name(cfg: int, w) -> str:
-    base = {0: "tiny dense top-5", 1: "paper-shaped dense top-5", 2: "clustered dense top-10",
-            3: "hybrid dense+BM25 top-5", 4: "scale dense top-100 with 4096-row upserts"}[cfg]
-    return f"{base}: {w.n} x {w.d} {w.dtype}, {w.q} queries/step"
-
-
-def roofline_terms(w, cfg):
-    """Algorithmic bytes and flops of one search-kernel launch."""
-    elem = 4 if w.dtype == "f32" else 2
-    corpus = w.n * w.d * elem
-    queries = w.q * w.d * elem
-    nbytes = corpus + queries
-    if cfg == 3:
-        nbytes += w.q * ((w.n + 3) // 4 * 4) * 4      # fused epilogue reads the BM25 block
-    flops = 2.0 * w.q * w.n * w.d
-    return nbytes, flops
-
-
-def peaks():
-    """(HBM GB/s, bf16 TFLOP/s burst, bf16 TFLOP/s sustained, source)."""
-    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
-    if os.path.exists(path):
-        with open(path) as f:
-            m = json.load(f)
-        return (float(m["hbm_gbs"]), float(m["bf16_tflops"]),
-                float(m.get("bf16_tflops_sustained", m["bf16_tflops"])), "measured")
-    return 6800.0, 1900.0, 1700.0, "fallback"
-
-
-def source_hash() -> str:
+def source_hash(read=None) -> str:
     h = hashlib.sha256()
     for name in KERNEL_SOURCES:
-        with open(os.path.join(ROOT, "paper_2608_08340_gb300", "csrc", name), "rb") as f:
-            h.update(f.read())
+        path = os.path.join(ROOT, "paper_2608_08340_gb300", "csrc", name)
+        text = read(name) if read else open(path, encoding="utf-8").read()
+        h.update(_code_only(text).encode())
     return h.hexdigest()[:16]
 
 

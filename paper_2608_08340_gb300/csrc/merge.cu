@@ -4,8 +4,9 @@
 // local candidates to the global top-k, done inside one GPU: the producers
 // are corpus slices instead of index shards.
 //
-// Many lists (more than 32 per query): one CTA per query runs the block merge
-// of merge.cuh.
+// Three merges by list count and k: one warp per query over at most 32
+// sorted lists (head by head), one warp per query over more lists when
+// k <= 16, and the block merge of merge.cuh (one CTA per query) otherwise.
 #include "merge.cuh"
 
 namespace oprag {
@@ -25,8 +26,7 @@ merge_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int qi = blockIdx.x;
   if (qi >= q) return;
-  merge_one_query<KP, false>(ls, qi, k, kMergeWarps, out_ids, out_scores, kth_out, levels_out,
-                             smem_keys);
+  merge_one_query<KP>(ls, qi, k, kMergeWarps, out_ids, out_scores, kth_out, levels_out, smem_keys);
 }
 
 template <int KP>

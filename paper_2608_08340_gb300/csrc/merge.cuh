@@ -35,10 +35,9 @@ __device__ __forceinline__ int merge_list_count(const ListSet& ls, int tile) {
   return np;
 }
 
-// Shared memory: (nw + 1) * 2 * KP keys.  kL2Only: read the lists through L2
-// only (for lists written by other SMs of the same grid).  All threads of the
-// CTA call this; it ends with a barrier, so the buffer can be reused.
-template <int KP, bool kL2Only>
+// Shared memory: (nw + 1) * 2 * KP keys.  All threads of the CTA call this;
+// it ends with a barrier, so the buffer can be reused.
+template <int KP>
 __device__ __forceinline__ void merge_one_query(const ListSet& ls, int qi, int k, int nw,
                                 int64_t* __restrict__ out_ids, float* __restrict__ out_scores,
                                 float* __restrict__ kth_out, float* __restrict__ levels_out,
@@ -65,8 +64,7 @@ __device__ __forceinline__ void merge_one_query(const ListSet& ls, int qi, int k
       key[u] = kEmptyKey;
       if (i < hi) {
         const int p = i / kl;
-        const uint64_t* a = base + p * list_step + (i - p * kl);
-        key[u] = kL2Only ? __ldcg(reinterpret_cast<const unsigned long long*>(a)) : *a;
+        key[u] = base[p * list_step + (i - p * kl)];
       }
     }
 #pragma unroll

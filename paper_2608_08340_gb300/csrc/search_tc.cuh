@@ -6,26 +6,28 @@
 //
 // Work decomposition.  Queries are cut into tiles of 128 (the MMA M side, one
 // query per TMEM lane) and the corpus into tiles of BN rows (the MMA N side).
-// A unit is (corpus tile t, query tile j), numbered u = t * QT + j, and CTA c
-// of a persistent grid of C CTAs takes units c, c + C, c + 2C, ...  All CTAs
-// therefore sweep the corpus together, each corpus tile being read by the QT
-// CTAs that need it at about the same time (one HBM read, QT - 1 L2 hits).
-// CTA c meets the query tiles j == c (mod g), g = gcd(C, QT); it keeps one
-// running top-K list per query for each of them ("slots") and leaves it as
-// partial list p = c / g of tile j for the merge kernel.
+// A unit is (query tile j, corpus tile t).  The corpus tiles are grouped into
+// windows that stay in L2; inside a window the units are ordered j-major and
+// cut into one contiguous share per CTA of the persistent grid (UnitSeq), so
+// all CTAs read inside the same window at the same time while each CTA meets
+// only one or two query tiles.  A CTA keeps one running top-K list per query
+// of each tile it meets and leaves it as one partial list of that tile for
+// the merge kernel (list slot = CTA offset from the first CTA of the tile).
 //
-// Roles (320 threads):
+// Roles (320 threads with two epilogue sets, 192 with one):
 //   warp 0, lane 0: TMA producer.  Per K block of 64 bf16 (one 128-byte
 //                   swizzle row) it loads the 128 x 64 query tile and the
 //                   BN x 64 corpus tile into a pipeline stage.
 //   warp 1        : allocates 2 x BN TMEM columns (two fp32 accumulators);
 //                   lane 0 issues tcgen05.mma (M = 128, N = BN, K = 16).
-//   warps 2..9    : epilogue, two sets of four warps, set s draining
-//                   accumulator s.  Each thread owns one query (one TMEM
-//                   lane), reads its BN scores with tcgen05.ld and filters
-//                   them against its running k-th best score.
+//   warps 2..     : epilogue, one or two sets of four warps; with two sets,
+//                   set s drains accumulator s.  Each thread owns one query
+//                   (one TMEM lane), reads its BN scores with tcgen05.ld and
+//                   filters them against a lower bound of that query's k-th
+//                   best score (its own list, the unit, and the bounds that
+//                   the other lists publish).
 // The two accumulators let the MMAs of one unit overlap the filtering of the
-// previous two.  Every mbarrier wait is bounded (see common.cuh).
+// previous one(s).  Every mbarrier wait is bounded (see common.cuh).
 #pragma once
 #include <cuda.h>
 
