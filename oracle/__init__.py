@@ -11,9 +11,12 @@ patterns; both are widened exactly to double inside the C code.
 
 Function -> paper passage:
   dense_scores / search   Sec. 3.2 (Op_retrieve) and the TopK display of Sec. 4.4
-  bm25                    Sec. 4.4 (inverted-postings BM25 with exact
-                          full-corpus semantics; textbook Okapi form)
+  bm25                    Sec. 4.4 (BM25 over the whole corpus with exact
+                          statistics; textbook Okapi form)
   hybrid_search           Sec. 4.4 weighted score fusion display
+  rerank /                dense-first hybrid policy, Sec. 4.1 Retrieval and
+  hybrid_dense_first      Sec. 5.5 (dense top-N, then the fusion over those
+                          candidates; BM25 maximum over the candidates)
   upsert                  Sec. 3.2 (Op_upsert), Sec. 4.1 (Upsert paragraph)
   round_bf16              storage precision of the index (IEEE RNE)
 """
@@ -65,10 +68,12 @@ def _load():
         lib.oracle_bm25.argtypes = [P, P, I64, I32, D, D, P, P, I32, P, P, P, I32]
         lib.oracle_hybrid_search.argtypes = [P, I32, I64, I32, P, I32, I32, P, P, I32, D, D,
                                              P, P, D, I64, P, P, P, I32]
+        lib.oracle_rerank.argtypes = [P, I32, I64, I32, P, I32, I32, P, P, I32, D, D,
+                                      P, P, P, I64, D, I64, P, P, I32]
         lib.oracle_upsert.argtypes = [P, I32, I64, I32, P, P, I32, I64]
         lib.oracle_round_bf16.argtypes = [P, I64, P]
         for name in ("oracle_dense_scores", "oracle_topk_rows", "oracle_search", "oracle_bm25",
-                     "oracle_hybrid_search", "oracle_upsert"):
+                     "oracle_hybrid_search", "oracle_rerank", "oracle_upsert"):
             getattr(lib, name).restype = ctypes.c_int
         lib.oracle_round_bf16.restype = None
         _lib = lib
@@ -173,6 +178,35 @@ def hybrid_search(E, Q, doc_indptr, doc_terms, vocab: int, q_indptr, q_terms, al
         "hybrid")
     hybrid_search.last_threads = used
     return ids, sc, mx
+
+
+def rerank(E, Q, cand, doc_indptr, doc_terms, vocab: int, q_indptr, q_terms, alpha: float,
+           kout: int, k1: float = 1.2, b: float = 0.75, nthreads: int = 0):
+    """Fused top-kout over given candidates (q x N chunk ids, -1 = none), the
+    BM25 maximum taken over the candidates: (ids, scores)."""
+    E, Q = _mat(E, "E"), _mat(Q, "Q")
+    dip, dt = _csr(doc_indptr, doc_terms)
+    qip, qt = _csr(q_indptr, q_terms)
+    cand = np.ascontiguousarray(cand, dtype=np.int64)
+    n, q = E.shape[0], Q.shape[0]
+    if dip.shape[0] != n + 1 or qip.shape[0] != q + 1 or cand.shape[0] != q:
+        raise ValueError("shapes do not match")
+    ids = np.empty((q, kout), np.int64)
+    sc = np.empty((q, kout), np.float64)
+    _check(_load().oracle_rerank(
+        _ptr(E), _code(E), n, E.shape[1], _ptr(Q), _code(Q), q, _ptr(dip), _ptr(dt), vocab,
+        k1, b, _ptr(qip), _ptr(qt), _ptr(cand), cand.shape[1], alpha, kout, _ptr(ids), _ptr(sc),
+        nthreads), "rerank")
+    return ids, sc
+
+
+def hybrid_dense_first(E, Q, doc_indptr, doc_terms, vocab: int, q_indptr, q_terms,
+                       alpha: float, n_cand: int, kout: int, k1: float = 1.2, b: float = 0.75,
+                       nthreads: int = 0):
+    """Dense-first hybrid: exact dense top-n_cand, then rerank of those: (ids, scores)."""
+    cand, _ = search(E, Q, n_cand, nthreads)
+    return rerank(E, Q, cand, doc_indptr, doc_terms, vocab, q_indptr, q_terms, alpha, kout,
+                  k1, b, nthreads)
 
 
 def upsert(E: np.ndarray, ids, rows) -> None:

@@ -21,15 +21,21 @@
  *                           chunk id asc) and truncation: Sec. 4.4 and Sec. 7
  *                           state that partial top-k selection must return the
  *                           same result as the full sort.
- *   oracle_bm25          -- Okapi BM25 by a document-wise scan (the "exact
- *                           full-corpus BM25 semantics" of Sec. 4.4 / Sec. 7;
- *                           the paper names BM25 but prints no formula, so the
+ *   oracle_bm25          -- Okapi BM25 by a document-wise scan (BM25 over the
+ *                           whole corpus with exact statistics, Sec. 4.4 /
+ *                           Sec. 7; the paper names BM25 but prints no formula, so the
  *                           textbook Okapi form with the non-negative idf
  *                           ln(1 + (N - df + 0.5)/(df + 0.5)) is used).
  *   oracle_hybrid_search -- weighted score fusion of Sec. 4.4:
  *                           score = w_d * s_dense + w_l * s_lex with
  *                           w_d = alpha, w_l = 1 - alpha and
  *                           s_lex = BM25 / max_d BM25 (per query), then TopK.
+ *   oracle_rerank        -- the lexical rerank of the dense-first hybrid
+ *                           policy (Sec. 4.1 Retrieval, Sec. 5.5): the same
+ *                           fusion restricted to given candidates (a dense
+ *                           top-N), with the BM25 maximum taken over those
+ *                           candidates (the paper does not say which maximum
+ *                           normalises a rerank; this is the reading used).
  *   oracle_upsert        -- Op_upsert of Sec. 3.2 (I' = Op_upsert(I, E; b_u)):
  *                           a literal row overwrite in the caller's order.
  *   oracle_round_bf16    -- fp32 -> bf16 round-to-nearest-even (the storage
@@ -388,6 +394,79 @@ int oracle_hybrid_search(const void *E, int edtype, int64_t n, int d,
     hybrid_ctx c = {&cs, E, edtype, d, Q, qdtype, q_indptr, q_terms, alpha, kout,
                     ids, scores, max_bm25, 0};
     int r = run_rows(hybrid_row, &c, q, 2 * n, nthreads);
+    free(cs.df);
+    return c.err ? -1 : r;
+}
+
+/* ------------------------------------------------------------ rerank */
+
+typedef struct {
+    const corpus_stats *cs;
+    const void *E; int edtype; int d;
+    const void *Q; int qdtype;
+    const int32_t *q_indptr; const int32_t *q_terms;
+    const int64_t *cand; int64_t ncand;
+    double alpha; int64_t kout;
+    int64_t *ids; double *scores; int err;
+} rerank_ctx;
+
+static void rerank_row(void *vctx, int64_t qi, double *work)
+{
+    (void)work;
+    rerank_ctx *c = (rerank_ctx *)vctx;
+    const int32_t *qt = c->q_terms + c->q_indptr[qi];
+    int nq = c->q_indptr[qi + 1] - c->q_indptr[qi];
+    const int64_t *cd = c->cand + qi * c->ncand;
+    pair_t *p = (pair_t *)malloc((size_t)(c->ncand > 0 ? c->ncand : 1) * sizeof(pair_t));
+    double *lex = (double *)malloc((size_t)(c->ncand > 0 ? c->ncand : 1) * sizeof(double));
+    if (!p || !lex) { free(p); free(lex); c->err = 1; return; }
+    /* BM25 of every candidate and the maximum over the candidates. */
+    int64_t m_valid = 0;
+    double m = 0.0;
+    for (int64_t i = 0; i < c->ncand; ++i) {
+        if (cd[i] < 0 || cd[i] >= c->cs->n) continue;
+        lex[i] = bm25_pair(c->cs, cd[i], qt, nq);
+        if (m_valid == 0 || lex[i] > m) m = lex[i];
+        ++m_valid;
+    }
+    int64_t np = 0;
+    for (int64_t i = 0; i < c->ncand; ++i) {
+        if (cd[i] < 0 || cd[i] >= c->cs->n) continue;
+        double dense = dot_row(c->E, c->edtype, cd[i], c->Q, c->qdtype, qi, c->d);
+        double lexn = m > 0.0 ? lex[i] / m : 0.0;
+        p[np].s = c->alpha * dense + (1.0 - c->alpha) * lexn;
+        p[np].id = cd[i];
+        ++np;
+    }
+    if (np < c->kout) { c->err = 1; free(p); free(lex); return; }
+    qsort(p, (size_t)np, sizeof(pair_t), pair_cmp);
+    for (int64_t i = 0; i < c->kout; ++i) {
+        c->ids[qi * c->kout + i] = p[i].id;
+        c->scores[qi * c->kout + i] = p[i].s;
+    }
+    free(p);
+    free(lex);
+}
+
+/* Rerank of given candidates (q x ncand chunk ids, -1 = none): fused top-kout
+ * of alpha * <q, e_d> + (1 - alpha) * BM25(q, d) / max over the candidates d'
+ * of BM25(q, d') (zero lexical part when that maximum is not positive).
+ * Every row needs at least kout candidates. */
+int oracle_rerank(const void *E, int edtype, int64_t n, int d,
+                  const void *Q, int qdtype, int q,
+                  const int32_t *doc_indptr, const int32_t *doc_terms, int vocab,
+                  double k1, double b,
+                  const int32_t *q_indptr, const int32_t *q_terms,
+                  const int64_t *cand, int64_t ncand,
+                  double alpha, int64_t kout,
+                  int64_t *ids, double *scores, int nthreads)
+{
+    if (kout < 0 || kout > ncand) return -1;
+    corpus_stats cs = {doc_indptr, doc_terms, n, vocab, k1, b, 0.0, NULL};
+    if (build_stats(&cs) != 0) return -1;
+    rerank_ctx c = {&cs, E, edtype, d, Q, qdtype, q_indptr, q_terms, cand, ncand, alpha, kout,
+                    ids, scores, 0};
+    int r = run_rows(rerank_row, &c, q, 0, nthreads);
     free(cs.df);
     return c.err ? -1 : r;
 }

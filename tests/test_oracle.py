@@ -259,6 +259,58 @@ def test_hybrid_alpha_zero_is_normalised_bm25_ranking():
         assert mx[i] == M[i].max()
 
 
+# ------------------------------------------------------------------ dense-first rerank
+
+def test_dense_first_golden_hand_worked():
+    g = load("dense_first_4doc.json")
+    h = load("hybrid_4doc.json")
+    bm = load("bm25_4doc.json")
+    dip, dt = _csr(bm["docs"])
+    qip, qt = _csr(h["query_terms"])
+    ids, sc = oracle.hybrid_dense_first(_f32(h["E"]), _f32(h["Q"]), dip, dt, bm["vocab"], qip,
+                                        qt, h["alpha"], g["n_cand"], g["k"], bm["k1"], bm["b"])
+    assert ids.tolist() == g["ids"]
+    want = np.array([[value(x) for x in row] for row in g["scores"]])
+    np.testing.assert_allclose(sc, want, rtol=0, atol=1e-15)
+    full, _, _ = oracle.hybrid_search(_f32(h["E"]), _f32(h["Q"]), dip, dt, bm["vocab"], qip, qt,
+                                      h["alpha"], 2, bm["k1"], bm["b"])
+    assert full.tolist() == g["full_hybrid_top2"]
+
+
+def test_rerank_over_every_chunk_is_the_full_hybrid():
+    w = _small_hybrid()
+    cand = np.tile(np.arange(w.n, dtype=np.int64), (w.q, 1))
+    ids, sc = oracle.rerank(w.E_data, w.Q_data, cand, w.doc_indptr, w.doc_terms, w.vocab,
+                            w.q_indptr, w.q_terms, w.alpha, 10, w.k1, w.b)
+    h_ids, h_sc, _ = oracle.hybrid_search(w.E_data, w.Q_data, w.doc_indptr, w.doc_terms, w.vocab,
+                                          w.q_indptr, w.q_terms, w.alpha, 10, w.k1, w.b)
+    np.testing.assert_array_equal(ids, h_ids)
+    np.testing.assert_allclose(sc, h_sc, rtol=0, atol=1e-12)
+
+
+def test_rerank_alpha_one_keeps_the_dense_order():
+    w = _small_hybrid()
+    ids, sc = oracle.hybrid_dense_first(w.E_data, w.Q_data, w.doc_indptr, w.doc_terms, w.vocab,
+                                        w.q_indptr, w.q_terms, 1.0, 32, 10, w.k1, w.b)
+    d_ids, d_sc = oracle.search(w.E_data, w.Q_data, 10)
+    np.testing.assert_array_equal(ids, d_ids)
+    np.testing.assert_array_equal(sc, d_sc)
+
+
+def test_rerank_ignores_candidate_order_and_empty_slots():
+    w = _small_hybrid()
+    cand, _ = oracle.search(w.E_data, w.Q_data, 40)
+    ids, sc = oracle.rerank(w.E_data, w.Q_data, cand, w.doc_indptr, w.doc_terms, w.vocab,
+                            w.q_indptr, w.q_terms, w.alpha, 8, w.k1, w.b)
+    rng = np.random.default_rng(3)
+    shuffled = np.array([rng.permutation(r) for r in cand])
+    padded = np.concatenate([shuffled, -np.ones((w.q, 7), np.int64)], axis=1)
+    ids2, sc2 = oracle.rerank(w.E_data, w.Q_data, padded, w.doc_indptr, w.doc_terms, w.vocab,
+                              w.q_indptr, w.q_terms, w.alpha, 8, w.k1, w.b)
+    np.testing.assert_array_equal(ids, ids2)
+    np.testing.assert_array_equal(sc, sc2)
+
+
 # ------------------------------------------------------------------ upsert
 
 def test_upsert_last_duplicate_wins_and_matches_rebuild():
