@@ -60,6 +60,60 @@ def source_hash(read=None) -> str:
     return h.hexdigest()[:16]
 
 
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--config", type=int, default=1)
+    p.add_argument("--batch", type=int, default=None)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--block-n", type=int, default=0, help="tensor-core tile rows (0 = auto)")
+    p.add_argument("--path", choices=["auto", "simt", "tc"], default="auto")
+    p.add_argument("--pair", choices=["auto", "single", "pair"], default="auto",
+                   help="tensor-core kernel: CTA pairs (M = 256 MMAs) or single CTAs")
+    p.add_argument("--dense-first", type=int, default=0, metavar="N",
+                   help="config 3 only: dense top-N, then the lexical rerank of those N "
+                        "candidates (dense-first hybrid) instead of the full hybrid")
+    return p.parse_args()
+
+
+def default_batch(cfg: int) -> int:
+    return {0: 16, 1: 256, 2: 4096, 3: 1024, 4: 2048}[cfg]
+
+
+def workload_name(cfg: int, w, dense_first: int = 0) -> str:
+    base = {0: "tiny dense top-5", 1: "paper-shaped dense top-5", 2: "clustered dense top-10",
+            3: "hybrid dense+BM25 top-5", 4: "scale dense top-100 with 4096-row upserts"}[cfg]
+    if cfg == 3 and dense_first:
+        base = f"dense-first hybrid top-5 (dense top-{dense_first}, lexical rerank)"
+    return f"{base}: {w.n} x {w.d} {w.dtype}, {w.q} queries/step"
+
+
+def roofline_terms(w, cfg, dense_first: int = 0):
+    """Algorithmic bytes and flops of one search-kernel launch."""
+    elem = 4 if w.dtype == "f32" else 2
+    corpus = w.n * w.d * elem
+    queries = w.q * w.d * elem
+    nbytes = corpus + queries
+    if cfg == 3 and not dense_first:
+        nbytes += w.q * ((w.n + 3) // 4 * 4) * 4      # fused epilogue reads the BM25 block
+    flops = 2.0 * w.q * w.n * w.d
+    return nbytes, flops
+
+
+def peaks():
+    """(HBM GB/s, bf16 TFLOP/s burst, bf16 TFLOP/s sustained, source)."""
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            m = json.load(f)
+        return (float(m["hbm_gbs"]), float(m["bf16_tflops"]),
+                float(m.get("bf16_tflops_sustained", m["bf16_tflops"])), "measured")
+    return 6800.0, 1900.0, 1700.0, "fallback"
+
+
 def ncu_traffic(workload_key: str):
     """DRAM bytes per launch of the dominant kernel from the committed ncu
     summary, if it was taken on the current kernel sources."""
@@ -220,6 +274,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
     cfg = args.config
+    dense_first = args.dense_first if cfg == 3 else 0
     batch = args.batch or default_batch(cfg)
     w = make_inputs(cfg, batch)
 
@@ -265,14 +320,18 @@ def run_ours(args, rank: int, world: int, local_rank: int):
             if cfg == 3:
                 raise RuntimeError("unreachable")
             idx.search_host(Qh, w.k, out=(ids_h, scores_h))
+        elif cfg == 3 and dense_first:
+            idx.hybrid_search_dense_first(Q, q_indptr, q_terms, w.alpha, dense_first, w.k)
         elif cfg == 3:
             idx.hybrid_search(Q, q_indptr, q_terms, w.alpha, w.k)
         else:
             idx.search(Q, w.k, out=(ids, scores))
 
     # search + merge; k > 32 adds the sampled first pass (search + merge);
-    # config 3 adds the BM25 pass, config 4 the upsert scatter.
-    launches_per_step = 2 + (2 if w.k > 32 else 0) + (1 if cfg in (3, 4) else 0)
+    # config 3 adds the BM25 pass (dense-first: the dense top-N search, with
+    # the sampled pass for N > 32, and the rerank), config 4 the upsert scatter.
+    k_search = dense_first if dense_first else w.k
+    launches_per_step = 2 + (2 if k_search > 32 else 0) + (1 if cfg in (3, 4) else 0)
 
     for i in range(args.warmup):
         flush.zero_()
@@ -338,7 +397,11 @@ def run_ours(args, rank: int, world: int, local_rank: int):
             Qd = Qh.to(dev, non_blocking=True)
             qi = torch.from_numpy(w.q_indptr).to(dev, non_blocking=True)
             qt = torch.from_numpy(w.q_terms).to(dev, non_blocking=True)
-            r_ids, r_sc = idx.hybrid_search(Qd, qi, qt, w.alpha, w.k)
+            if dense_first:
+                r_ids, r_sc = idx.hybrid_search_dense_first(Qd, qi, qt, w.alpha, dense_first,
+                                                            w.k)
+            else:
+                r_ids, r_sc = idx.hybrid_search(Qd, qi, qt, w.alpha, w.k)
             ids_h.copy_(r_ids)
             scores_h.copy_(r_sc)
             torch.cuda.synchronize()
@@ -354,7 +417,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
     if rank != 0:
         return None
 
-    nbytes, flops = roofline_terms(w, cfg)
+    nbytes, flops = roofline_terms(w, cfg, dense_first)
     hbm, tflops_burst, tflops_sustained, peak_src = peaks()
     # The burst figure is for a kernel timed alone; when the timed loop kept
     # the GPU at its power cap (NVML reported sw_power_cap while it ran), the
@@ -399,18 +462,32 @@ def run_ours(args, rank: int, world: int, local_rank: int):
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": total_ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-        "config": {"workload": workload_name(cfg, w), "config_index": cfg, "n": w.n, "d": w.d,
-                   "q": w.q, "k": w.k, "parallelism": f"replicas{world}",
+        "config": {"workload": workload_name(cfg, w, dense_first), "config_index": cfg,
+                   "n": w.n, "d": w.d, "q": w.q, "k": w.k, "parallelism": f"replicas{world}",
                    "l2": f"flushed before every step ({L2_FLUSH_BYTES >> 20} MiB write)"},
         "roofline": roof,
         "e2e": {"value": queries_all / (e2e_total * 1e-3), "unit": "queries/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                "api": "oprag_search_host" if cfg != 3 else "oprag_hybrid_search + torch copies"},
+                "api": ("oprag_search_host" if cfg != 3 else
+                        "oprag_hybrid_search_dense_first + torch copies" if dense_first else
+                        "oprag_hybrid_search + torch copies")},
         "gpu_launches": launches_per_step * args.steps,
         "clocks": dict(clocks.summary(), smi=smi.summary()),
         "path": idx.last_path,
         "launch": idx.last_launch,
     }
+    if dense_first:
+        # Quality against the full hybrid search (Sec. 5.2 Recall@k; Jaccard
+        # overlap of the two top-k sets), as the paper reports for this policy.
+        f_ids, _ = idx.hybrid_search(Q, q_indptr, q_terms, w.alpha, w.k)
+        d_ids, _ = idx.hybrid_search_dense_first(Q, q_indptr, q_terms, w.alpha, dense_first, w.k)
+        f_ids, d_ids = f_ids.cpu().numpy(), d_ids.cpu().numpy()
+        inter = [len(set(a) & set(b)) for a, b in zip(f_ids.tolist(), d_ids.tolist())]
+        union = [len(set(a) | set(b)) for a, b in zip(f_ids.tolist(), d_ids.tolist())]
+        result["quality"] = {"recall_at_k": float(np.mean(inter)) / w.k,
+                             "jaccard": float(np.mean([i / u for i, u in zip(inter, union)])),
+                             "vs": "full hybrid search on the same batch",
+                             "n_candidates": dense_first}
     idx.close()
     return result, w
 

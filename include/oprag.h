@@ -164,6 +164,24 @@ OPRAG_API int oprag_hybrid_search(oprag_index *idx, const void *queries, int32_t
                         float *out_scores, void *stream);
 
 /*
+ * Dense-first hybrid search (Sec. 4.1 Retrieval; Sec. 5.5): the exact dense
+ * top-n_cand of each query (as oprag_search), then the fusion of
+ * oprag_hybrid_search applied only to those candidates, with the BM25
+ * maximum taken over the candidates (the paper does not name the maximum of a
+ * rerank), and the top-k of the fused scores (score descending, chunk id
+ * ascending).  With every chunk a candidate (n_cand >= n) the result equals
+ * oprag_hybrid_search.
+ *   queries, q_indptr, q_terms, alpha   as oprag_hybrid_search (device).
+ *   n_cand       candidates per query, k <= n_cand <= 256 (fewer when n < n_cand).
+ *   out_ids / out_scores   device, q x k.
+ * Asynchronous on `stream`.  OPRAG_ERR_NOT_READY without a sparse side.
+ */
+OPRAG_API int oprag_hybrid_search_dense_first(oprag_index *idx, const void *queries, int32_t q,
+                                              const int32_t *q_indptr, const int32_t *q_terms,
+                                              float alpha, int32_t n_cand, int32_t k,
+                                              int64_t *out_ids, float *out_scores, void *stream);
+
+/*
  * Waits for the index's pending work and reports whether a kernel of it gave
  * up a bounded wait since the last check (OPRAG_ERR_DEVICE; the flag is then
  * cleared) or a CUDA error occurred (OPRAG_ERR_CUDA).

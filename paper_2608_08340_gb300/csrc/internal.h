@@ -127,6 +127,15 @@ cudaError_t launch_bm25_matrix(const SparseIndex& sp, int64_t n, const int32_t* 
                                const int32_t* q_terms, int q, float* out, int64_t ld,
                                float* out_max, cudaStream_t st);
 
+// --- lexical rerank of a dense top-N (dense-first hybrid), rerank.cu.
+// cand_ids / cand_scores: q x ncand dense results (id -1 = none), ncand <=
+// kRerankMaxCand; writes the fused top-k (k <= ncand) of each query.
+constexpr int kRerankMaxCand = 256;
+cudaError_t launch_rerank(const SparseIndex& sp, int q, int ncand, const int64_t* cand_ids,
+                          const float* cand_scores, const int32_t* q_indptr,
+                          const int32_t* q_terms, float alpha, int k, int64_t* out_ids,
+                          float* out_scores, cudaStream_t st);
+
 // --- upsert / conversion.
 cudaError_t launch_scatter_rows(int index_dtype, void* E, int d, const void* rows, int rows_dtype,
                                 const int64_t* src_dst /* pairs: source row, destination row */,

@@ -76,6 +76,8 @@ struct oprag_index {
   size_t scratch_bytes = 0;
   float* lex = nullptr;        // BM25 block (q x ld) followed by q maxima
   size_t lex_bytes = 0;
+  void* cand = nullptr;        // dense-first candidates: q x N ids, then q x N scores
+  size_t cand_bytes = 0;
   void* stage = nullptr;       // upsert staging / host-buffer search staging
   size_t stage_bytes = 0;
 
@@ -396,6 +398,7 @@ void oprag_index_destroy(oprag_index* idx) {
   if (idx->scratch) cudaFree(idx->scratch);
   if (idx->qfloor) cudaFree(idx->qfloor);
   if (idx->lex) cudaFree(idx->lex);
+  if (idx->cand) cudaFree(idx->cand);
   if (idx->stage) cudaFree(idx->stage);
   idx->free_sparse();
   if (idx->done) cudaEventDestroy(idx->done);
@@ -694,6 +697,41 @@ int oprag_hybrid_search(oprag_index* idx, const void* queries, int32_t q, const 
                          out_scores + static_cast<size_t>(c0) * k, st)))
       return rc;
   }
+  return end_call(idx, st);
+}
+
+int oprag_hybrid_search_dense_first(oprag_index* idx, const void* queries, int32_t q,
+                                    const int32_t* q_indptr, const int32_t* q_terms, float alpha,
+                                    int32_t n_cand, int32_t k, int64_t* out_ids,
+                                    float* out_scores, void* stream) {
+  int rc = check_search_args(idx, queries, q, k, out_ids, out_scores);
+  if (rc) return rc;
+  if (!idx->has_sparse) return fail(OPRAG_ERR_NOT_READY, "no sparse side: call oprag_index_set_sparse");
+  if (n_cand < k || n_cand > kRerankMaxCand)
+    return fail(OPRAG_ERR_INVALID_ARG, "need k <= n_cand <= %d (n_cand = %d, k = %d)",
+                kRerankMaxCand, n_cand, k);
+  if (q == 0) return ok();
+  if (!q_indptr || !q_terms) return fail(OPRAG_ERR_INVALID_ARG, "NULL query terms");
+  if (!std::isfinite(alpha)) return fail(OPRAG_ERR_INVALID_ARG, "alpha is not finite");
+  // A corpus smaller than n_cand gives every chunk as a candidate.
+  const int nc = static_cast<int>(std::min<int64_t>(n_cand, idx->n));
+  DeviceGuard g(idx->device);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t ids_bytes = static_cast<size_t>(q) * nc * sizeof(int64_t);
+  if ((rc = idx->ensure(&idx->cand, &idx->cand_bytes,
+                        ids_bytes + static_cast<size_t>(q) * nc * sizeof(float),
+                        "dense-first candidates")))
+    return rc;
+  if ((rc = begin_call(idx, st))) return rc;
+  int64_t* cid = static_cast<int64_t*>(idx->cand);
+  float* csc = reinterpret_cast<float*>(static_cast<char*>(idx->cand) + ids_bytes);
+  const Fusion none{nullptr, 0, nullptr, 0.f};
+  if ((rc = run_search(idx, queries, q, nc, none, cid, csc, st))) return rc;
+  const SparseIndex sp{idx->vocab,      idx->nnz,     idx->post_ptr, idx->post,
+                       idx->dense_slot, idx->dense_w, idx->dense_ld};
+  cudaError_t e = launch_rerank(sp, q, nc, cid, csc, q_indptr, q_terms, alpha, k, out_ids,
+                                out_scores, st);
+  if (e != cudaSuccess) return cuda_fail(e, "rerank kernel");
   return end_call(idx, st);
 }
 

@@ -133,6 +133,26 @@ class Index:
                                             _stream_ptr(stream)))
         return ids, scores
 
+    def hybrid_search_dense_first(self, queries: torch.Tensor, q_indptr: torch.Tensor,
+                                  q_terms: torch.Tensor, alpha: float, n_cand: int, k: int,
+                                  stream=None):
+        """Dense top-n_cand, then the fused rerank of those candidates (BM25
+        maximum over the candidates); top-k (ids, scores)."""
+        queries = self._queries(queries)
+        q = int(queries.shape[0])
+        qip = q_indptr.to(device=queries.device, dtype=torch.int32).contiguous()
+        qt = q_terms.to(device=queries.device, dtype=torch.int32).contiguous()
+        if qt.numel() == 0:
+            qt = torch.zeros(1, dtype=torch.int32, device=queries.device)
+        if qip.numel() != q + 1:
+            raise ValueError("q_indptr must have q + 1 entries")
+        ids = torch.empty((q, k), dtype=torch.int64, device=queries.device)
+        scores = torch.empty((q, k), dtype=torch.float32, device=queries.device)
+        check(self._lib.oprag_hybrid_search_dense_first(
+            self._h, _ptr(queries), q, _ptr(qip), _ptr(qt), float(alpha), n_cand, k, _ptr(ids),
+            _ptr(scores), _stream_ptr(stream)))
+        return ids, scores
+
     # -- upsert
     def upsert(self, ids, rows: torch.Tensor, stream=None) -> None:
         """rows[i] overwrites chunk ids[i] (host int64 ids; later duplicates win)."""
