@@ -17,6 +17,8 @@ Function -> paper passage:
   rerank /                dense-first hybrid policy, Sec. 4.1 Retrieval and
   hybrid_dense_first      Sec. 5.5 (dense top-N, then the fusion over those
                           candidates; BM25 maximum over the candidates)
+  embed_pool              Sec. 4.3 (hidden states -> mean pool -> L2 normalise;
+                          padded positions masked)
   upsert                  Sec. 3.2 (Op_upsert), Sec. 4.1 (Upsert paragraph)
   round_bf16              storage precision of the index (IEEE RNE)
 """
@@ -70,10 +72,12 @@ def _load():
                                              P, P, D, I64, P, P, P, I32]
         lib.oracle_rerank.argtypes = [P, I32, I64, I32, P, I32, I32, P, P, I32, D, D,
                                       P, P, P, I64, D, I64, P, P, I32]
+        lib.oracle_embed_pool.argtypes = [P, I32, I32, I32, I32, P, P]
         lib.oracle_upsert.argtypes = [P, I32, I64, I32, P, P, I32, I64]
         lib.oracle_round_bf16.argtypes = [P, I64, P]
         for name in ("oracle_dense_scores", "oracle_topk_rows", "oracle_search", "oracle_bm25",
-                     "oracle_hybrid_search", "oracle_rerank", "oracle_upsert"):
+                     "oracle_hybrid_search", "oracle_rerank", "oracle_embed_pool",
+                     "oracle_upsert"):
             getattr(lib, name).restype = ctypes.c_int
         lib.oracle_round_bf16.restype = None
         _lib = lib
@@ -207,6 +211,23 @@ def hybrid_dense_first(E, Q, doc_indptr, doc_terms, vocab: int, q_indptr, q_term
     cand, _ = search(E, Q, n_cand, nthreads)
     return rerank(E, Q, cand, doc_indptr, doc_terms, vocab, q_indptr, q_terms, alpha, kout,
                   k1, b, nthreads)
+
+
+def embed_pool(hidden, mask):
+    """batch x dim fp64: masked mean over tokens, then L2 normalisation.
+    hidden: batch x tokens x dim, float32 or uint16 (bf16 bits); mask:
+    batch x tokens, nonzero = a real token."""
+    h = np.ascontiguousarray(hidden)
+    _code(h)
+    if h.ndim != 3:
+        raise ValueError("hidden must be 3-D")
+    m = np.ascontiguousarray(mask, dtype=np.uint8)
+    if m.shape != h.shape[:2]:
+        raise ValueError("mask must be batch x tokens")
+    out = np.empty((h.shape[0], h.shape[2]), np.float64)
+    _check(_load().oracle_embed_pool(_ptr(h), _code(h), h.shape[0], h.shape[1], h.shape[2],
+                                     _ptr(m), _ptr(out)), "embed_pool")
+    return out
 
 
 def upsert(E: np.ndarray, ids, rows) -> None:

@@ -36,6 +36,10 @@
  *                           top-N), with the BM25 maximum taken over those
  *                           candidates (the paper does not say which maximum
  *                           normalises a rerank; this is the reading used).
+ *   oracle_embed_pool    -- the tail of Op_embed (Sec. 4.3: hidden states of
+ *                           a chunk -> mean pool -> L2 normalise), with the
+ *                           padded token positions of a batch masked out
+ *                           (length-bucketed batches are padded, Sec. 4.3).
  *   oracle_upsert        -- Op_upsert of Sec. 3.2 (I' = Op_upsert(I, E; b_u)):
  *                           a literal row overwrite in the caller's order.
  *   oracle_round_bf16    -- fp32 -> bf16 round-to-nearest-even (the storage
@@ -469,6 +473,38 @@ int oracle_rerank(const void *E, int edtype, int64_t n, int d,
     int r = run_rows(rerank_row, &c, q, 0, nthreads);
     free(cs.df);
     return c.err ? -1 : r;
+}
+
+/* ------------------------------------------------------------ embedding tail */
+
+/* out[b] = m / ||m|| with m = (1 / c) * sum of hidden[b][t] over the c tokens t
+ * with mask[b][t] != 0 (hidden is batch x tokens x dim, fp32 or bf16 bits).
+ * A row with no unmasked token or a zero mean gives a zero vector. */
+int oracle_embed_pool(const void *hidden, int hdtype, int batch, int tokens, int dim,
+                      const uint8_t *mask, double *out)
+{
+    if (batch < 0 || tokens < 0 || dim <= 0) return -1;
+    for (int b = 0; b < batch; ++b) {
+        double *o = out + (int64_t)b * dim;
+        for (int j = 0; j < dim; ++j) o[j] = 0.0;
+        int64_t c = 0;
+        for (int t = 0; t < tokens; ++t) {
+            if (!mask[(int64_t)b * tokens + t]) continue;
+            ++c;
+            int64_t row = ((int64_t)b * tokens + t) * dim;
+            for (int j = 0; j < dim; ++j) o[j] += load_elem(hidden, hdtype, row + j);
+        }
+        if (c == 0) continue;
+        double ss = 0.0;
+        for (int j = 0; j < dim; ++j) {
+            o[j] /= (double)c;
+            ss += o[j] * o[j];
+        }
+        if (ss == 0.0) continue;
+        double norm = sqrt(ss);
+        for (int j = 0; j < dim; ++j) o[j] /= norm;
+    }
+    return 0;
 }
 
 /* ------------------------------------------------------------ upsert */

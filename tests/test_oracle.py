@@ -311,6 +311,56 @@ def test_rerank_ignores_candidate_order_and_empty_slots():
     np.testing.assert_array_equal(sc, sc2)
 
 
+# ------------------------------------------------------------------ embedding tail
+
+def test_embed_pool_golden_hand_worked():
+    g = load("embed_pool_2tok.json")
+    out = oracle.embed_pool(np.array(g["hidden"], np.float32), np.array(g["mask"], np.uint8))
+    want = np.array([[value(x) for x in row] for row in g["normalised_exact"]])
+    np.testing.assert_allclose(out, want, rtol=0, atol=1e-15)
+    bits = oracle.round_bf16(out.astype(np.float32))
+    assert bits.tolist() == g["bf16_bits"]
+
+
+def test_embed_pool_single_token_and_identical_tokens_are_the_normalised_token():
+    rng = np.random.default_rng(7)
+    h = rng.standard_normal((5, 6, 64)).astype(np.float32)
+    mask = np.zeros((5, 6), np.uint8)
+    mask[:, 2] = 1
+    out = oracle.embed_pool(h, mask)
+    tok = h[:, 2, :].astype(np.float64)
+    np.testing.assert_allclose(out, tok / np.linalg.norm(tok, axis=1, keepdims=True), atol=1e-15)
+    same = np.repeat(h[:, :1, :], 6, axis=1)
+    np.testing.assert_allclose(oracle.embed_pool(same, np.ones((5, 6), np.uint8)),
+                               oracle.embed_pool(same[:, :1, :], np.ones((5, 1), np.uint8)),
+                               atol=1e-15)
+
+
+def test_embed_pool_is_a_unit_vector_invariant_to_scale_and_masked_values():
+    rng = np.random.default_rng(8)
+    h = rng.standard_normal((4, 9, 48)).astype(np.float32)
+    mask = (rng.random((4, 9)) < 0.6).astype(np.uint8)
+    mask[:, 0] = 1
+    out = oracle.embed_pool(h, mask)
+    np.testing.assert_allclose(np.linalg.norm(out, axis=1), 1.0, atol=1e-14)
+    np.testing.assert_allclose(oracle.embed_pool(h * np.float32(4.0), mask), out, atol=1e-14)
+    h2 = h.copy()
+    h2[mask == 0] = 1e3                                   # padding values do not matter
+    np.testing.assert_array_equal(oracle.embed_pool(h2, mask), out)
+    # the mean of the unmasked tokens, written out with numpy
+    m = np.stack([h[b][mask[b] == 1].astype(np.float64).mean(axis=0) for b in range(4)])
+    np.testing.assert_allclose(out, m / np.linalg.norm(m, axis=1, keepdims=True), atol=1e-14)
+
+
+def test_embed_pool_bf16_input_widens_exactly():
+    rng = np.random.default_rng(9)
+    h = rng.standard_normal((3, 4, 32)).astype(np.float32)
+    bits = oracle.round_bf16(h)
+    widened = oracle.bf16_to_f32(bits)
+    mask = np.ones((3, 4), np.uint8)
+    np.testing.assert_array_equal(oracle.embed_pool(bits, mask), oracle.embed_pool(widened, mask))
+
+
 # ------------------------------------------------------------------ upsert
 
 def test_upsert_last_duplicate_wins_and_matches_rebuild():
