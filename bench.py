@@ -73,6 +73,9 @@ def parse():
     p.add_argument("--path", choices=["auto", "simt", "tc"], default="auto")
     p.add_argument("--pair", choices=["auto", "single", "pair"], default="auto",
                    help="tensor-core kernel: CTA pairs (M = 256 MMAs) or single CTAs")
+    p.add_argument("--embed-tail", action="store_true",
+                   help="time the embedding tail instead (masked mean pool + L2 normalise of "
+                        "256 x 512 x 4096 bf16 hidden states, the Llama3-8B hidden size)")
     p.add_argument("--dense-first", type=int, default=0, metavar="N",
                    help="config 3 only: dense top-N, then the lexical rerank of those N "
                         "candidates (dense-first hybrid) instead of the full hybrid")
@@ -558,8 +561,55 @@ def run_reference(args):
     print(json.dumps(out))
 
 
+def run_embed_tail(args):
+    """Embedding tail (Sec. 4.3): rows/s and HBM roofline of oprag_embed_pool on a
+    synthetic padded batch (lengths uniform in [T/4, T])."""
+    import torch
+    from paper_2608_08340_gb300.index import embed_pool
+
+    torch.cuda.set_device(0)
+    b, t, d = 256, 512, 4096
+    g = torch.Generator(device="cuda").manual_seed(5000)
+    hidden = torch.randn((b, t, d), generator=g, device="cuda").to(torch.bfloat16)
+    rng = np.random.default_rng(5001)
+    lens = rng.integers(t // 4, t + 1, b)
+    mask = torch.from_numpy((np.arange(t)[None, :] < lens[:, None]).astype(np.uint8)).cuda()
+    for _ in range(args.warmup):
+        embed_pool(hidden, mask)
+    torch.cuda.synchronize()
+    marks = []
+    for _ in range(args.steps):
+        a = torch.cuda.Event(enable_timing=True)
+        e = torch.cuda.Event(enable_timing=True)
+        a.record()
+        embed_pool(hidden, mask)
+        e.record()
+        marks.append((a, e))
+    torch.cuda.synchronize()
+    ms = [a.elapsed_time(e) for a, e in marks]
+    t_step = statistics.mean(ms) * 1e-3
+    # bytes the kernel must move: the unmasked hidden states, the mask, the output
+    nbytes = int(lens.sum()) * d * 2 + b * t + b * d * 2
+    hbm = peaks()[0]
+    print(json.dumps({
+        "metric": "embedded rows/s (masked mean pool + L2 normalise)", "value": b / t_step,
+        "unit": "rows/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": statistics.mean(ms), "higher_is_better": True, "dtype": "bf16",
+        "data": "synthetic", "scaling": "weak", "vs_baseline": None,
+        "config": {"workload": f"embedding tail: {b} rows x {t} tokens x {d} bf16, lengths "
+                               f"uniform in [{t // 4}, {t}]",
+                   "l2": "input (1 GiB) larger than L2"},
+        "roofline": {"bound": "hbm", "achieved": nbytes / t_step / 1e9, "peak": hbm,
+                     "unit": "GB/s", "frac": nbytes / t_step / 1e9 / hbm,
+                     "algorithmic_bytes": nbytes, "kernel": "embed_pool_kernel"},
+        "gpu_launches": args.steps}))
+
+
 def main():
     args = parse()
+    if args.embed_tail and args.impl == "ours":
+        run_embed_tail(args)
+        return
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))

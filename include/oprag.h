@@ -182,6 +182,24 @@ OPRAG_API int oprag_hybrid_search_dense_first(oprag_index *idx, const void *quer
                                               int64_t *out_ids, float *out_scores, void *stream);
 
 /*
+ * Tail of Op_embed (Sec. 4.3: hidden states -> mean pool -> L2 normalise), for
+ * a padded batch of chunks or queries:
+ *   out[b] = m / ||m||,  m = (1 / c) * sum of hidden[b][t] over the c tokens t
+ *   with mask[b][t] != 0  (a row with c = 0 or m = 0 gives zeros).
+ *   hidden      device, batch x tokens x dim, OPRAG_BF16 or OPRAG_F32
+ *               (hidden_dtype), 16-byte aligned; dim a multiple of 8, at most
+ *               16384 (bf16) or 8192 (fp32).
+ *   mask        device, batch x tokens uint8 (nonzero = a real token).
+ *   out         device, batch x dim in out_dtype (OPRAG_BF16: round to nearest
+ *               even of the fp32 result), 16-byte aligned; as queries it feeds
+ *               oprag_search of an index of the same dim directly.
+ * Accumulates in fp32.  Asynchronous on `stream`; needs no index.
+ */
+OPRAG_API int oprag_embed_pool(const void *hidden, int32_t hidden_dtype, int32_t batch,
+                               int32_t tokens, int32_t dim, const uint8_t *mask, void *out,
+                               int32_t out_dtype, void *stream);
+
+/*
  * Waits for the index's pending work and reports whether a kernel of it gave
  * up a bounded wait since the last check (OPRAG_ERR_DEVICE; the flag is then
  * cleared) or a CUDA error occurred (OPRAG_ERR_CUDA).

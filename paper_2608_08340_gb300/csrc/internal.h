@@ -136,6 +136,12 @@ cudaError_t launch_rerank(const SparseIndex& sp, int q, int ncand, const int64_t
                           const int32_t* q_terms, float alpha, int k, int64_t* out_ids,
                           float* out_scores, cudaStream_t st);
 
+// --- embedding tail (embed.cu): masked mean pool + L2 normalisation of a
+// batch x tokens x dim block of hidden states into batch x dim vectors.
+// dim % 8 == 0 and dim <= 16384 (bf16 input) / 8192 (fp32 input).
+cudaError_t launch_embed_pool(int hidden_dtype, const void* hidden, int batch, int tokens, int dim,
+                              const uint8_t* mask, int out_dtype, void* out, cudaStream_t st);
+
 // --- upsert / conversion.
 cudaError_t launch_scatter_rows(int index_dtype, void* E, int d, const void* rows, int rows_dtype,
                                 const int64_t* src_dst /* pairs: source row, destination row */,

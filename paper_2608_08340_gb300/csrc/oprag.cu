@@ -735,6 +735,28 @@ int oprag_hybrid_search_dense_first(oprag_index* idx, const void* queries, int32
   return end_call(idx, st);
 }
 
+int oprag_embed_pool(const void* hidden, int32_t hidden_dtype, int32_t batch, int32_t tokens,
+                     int32_t dim, const uint8_t* mask, void* out, int32_t out_dtype,
+                     void* stream) {
+  if (hidden_dtype != OPRAG_F32 && hidden_dtype != OPRAG_BF16)
+    return fail(OPRAG_ERR_INVALID_ARG, "hidden dtype %d", hidden_dtype);
+  if (out_dtype != OPRAG_F32 && out_dtype != OPRAG_BF16)
+    return fail(OPRAG_ERR_INVALID_ARG, "output dtype %d", out_dtype);
+  if (batch < 0 || tokens < 1 || dim < 8 || dim % 8 != 0)
+    return fail(OPRAG_ERR_INVALID_ARG, "need batch >= 0, tokens >= 1, dim a positive multiple of 8");
+  if (dim > (hidden_dtype == OPRAG_BF16 ? 16384 : 8192))
+    return fail(OPRAG_ERR_INVALID_ARG, "dim %d too large", dim);
+  if (batch == 0) return ok();
+  if (!hidden || !mask || !out) return fail(OPRAG_ERR_INVALID_ARG, "NULL argument");
+  if ((reinterpret_cast<uintptr_t>(hidden) | reinterpret_cast<uintptr_t>(out)) % 16 != 0)
+    return fail(OPRAG_ERR_INVALID_ARG, "hidden and out must be 16-byte aligned");
+  cudaError_t e = launch_embed_pool(hidden_dtype == OPRAG_BF16 ? kBF16 : kF32, hidden, batch,
+                                    tokens, dim, mask, out_dtype == OPRAG_BF16 ? kBF16 : kF32, out,
+                                    static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail(e, "embedding tail kernel");
+  return ok();
+}
+
 int oprag_index_check(oprag_index* idx) {
   if (!idx) return fail(OPRAG_ERR_INVALID_ARG, "index is NULL");
   DeviceGuard g(idx->device);

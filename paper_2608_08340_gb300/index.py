@@ -214,3 +214,27 @@ class Index:
     @property
     def last_path(self) -> str:
         return {0: "none", 1: "simt", 2: "tc"}[self._lib.oprag_index_last_path(self._h)]
+
+
+def embed_pool(hidden: torch.Tensor, mask: torch.Tensor, out_dtype: torch.dtype = torch.bfloat16,
+               stream=None) -> torch.Tensor:
+    """Tail of Op_embed: masked mean pool over tokens, then L2 normalisation.
+
+    hidden: (batch, tokens, dim) bfloat16 or float32 CUDA tensor; mask:
+    (batch, tokens) bool or uint8 (nonzero = a real token).  Returns
+    (batch, dim) in out_dtype (bfloat16 or float32), usable as queries."""
+    lib = _lib.load()
+    if hidden.dim() != 3 or hidden.dtype not in _DT or not hidden.is_cuda:
+        raise ValueError("hidden must be a 3-D bfloat16 or float32 CUDA tensor")
+    if out_dtype not in _DT:
+        raise ValueError("out_dtype must be bfloat16 or float32")
+    b, t, d = (int(x) for x in hidden.shape)
+    hidden = hidden.contiguous()
+    m = mask.to(device=hidden.device, dtype=torch.uint8).contiguous()
+    if tuple(m.shape) != (b, t):
+        raise ValueError("mask must be (batch, tokens)")
+    out = torch.empty((b, d), dtype=out_dtype, device=hidden.device)
+    check(lib.oprag_embed_pool(_ptr(hidden), _DT[hidden.dtype], b, t, d, _ptr(m), _ptr(out),
+                               _DT[out_dtype], _stream_ptr(stream)))
+    return out
+
