@@ -20,6 +20,8 @@ Function -> paper passage:
   embed_pool              Sec. 4.3 (hidden states -> mean pool -> L2 normalise;
                           padded positions masked)
   upsert                  Sec. 3.2 (Op_upsert), Sec. 4.1 (Upsert paragraph)
+  replace_bags            the lexical half of Op_upsert (Sec. 3.2, Sec. 4.4)
+  search_two              knowledge + memory index, one ranked result (Sec. 4.4)
   round_bf16              storage precision of the index (IEEE RNE)
 """
 from __future__ import annotations
@@ -228,6 +230,41 @@ def embed_pool(hidden, mask):
     _check(_load().oracle_embed_pool(_ptr(h), _code(h), h.shape[0], h.shape[1], h.shape[2],
                                      _ptr(m), _ptr(out)), "embed_pool")
     return out
+
+
+def replace_bags(doc_indptr, doc_terms, ids, bag_indptr, bag_terms):
+    """Token bags after replacing those of chunks ids[i] by bag i (a later
+    duplicate id wins; ids at n.. append chunks, with empty bags for any chunk
+    between n and the largest id): (indptr, terms) of the new CSR.  The
+    lexical half of Op_upsert (Sec. 3.2; Sec. 4.4 keeps BM25 exact over the
+    corpus, so df and avgdl follow the new bags)."""
+    dip, dt = _csr(doc_indptr, doc_terms)
+    bip, bt = _csr(bag_indptr, bag_terms)
+    ids = np.asarray(ids, dtype=np.int64)
+    n = dip.shape[0] - 1
+    if ids.size and ids.min() < 0:
+        raise ValueError("negative chunk id")
+    n_new = max(n, int(ids.max()) + 1 if ids.size else n)
+    bags = [list(dt[dip[i]:dip[i + 1]]) for i in range(n)] + [[] for _ in range(n_new - n)]
+    for i, c in enumerate(ids.tolist()):
+        bags[c] = list(bt[bip[i]:bip[i + 1]])
+    ip = np.zeros(n_new + 1, np.int32)
+    ip[1:] = np.cumsum([len(b) for b in bags])
+    terms = np.array([t for b in bags for t in b], np.int32)
+    return ip, terms
+
+
+def search_two(Ek, Em, Q, kout: int, nthreads: int = 0):
+    """Top-kout over two indices (knowledge index Ek, memory index Em, Sec. 4.4:
+    both searched the same way, one ranked result): (ids, src, scores) where
+    src 0 = Ek, 1 = Em; order score descending, then src, then chunk id."""
+    nk = Ek.shape[0]
+    both = np.concatenate([np.ascontiguousarray(Ek), np.ascontiguousarray(Em)], axis=0)
+    # On the stacked matrix the (score desc, row asc) order is exactly
+    # (score desc, src asc, id asc).
+    ids, sc = search(both, Q, kout, nthreads)
+    src = (ids >= nk).astype(np.int32)
+    return np.where(src == 1, ids - nk, ids), src, sc
 
 
 def upsert(E: np.ndarray, ids, rows) -> None:

@@ -361,6 +361,41 @@ def test_embed_pool_bf16_input_widens_exactly():
     np.testing.assert_array_equal(oracle.embed_pool(bits, mask), oracle.embed_pool(widened, mask))
 
 
+# ------------------------------------------------------------------ bags, two indices
+
+def test_replace_bags_last_duplicate_wins_appends_and_recomputes_bm25():
+    g = load("bm25_4doc.json")
+    dip, dt = _csr(g["docs"])
+    # doc 1 becomes [4], doc 1 again (wins) becomes [5, 5], doc 5 appended (doc 4 empty)
+    ip, tm = oracle.replace_bags(dip, dt, [1, 1, 5], [0, 1, 3, 4], [4, 5, 5, 0])
+    assert ip.tolist() == [0, 2, 4, 7, 10, 10, 11]
+    assert tm.tolist() == [0, 1, 5, 5, 1, 2, 4, 3, 3, 3, 0]
+    # BM25 of term 0 on the new corpus, by hand: N = 6, df(0) = 2 (docs 0 and 5),
+    # lengths 2, 2, 3, 3, 0, 1 -> avgdl = 11/6; doc 0: tf 1, L = 1/4 + 3/4 * 2 / (11/6)
+    M, avgdl, df = oracle.bm25(ip, tm, g["vocab"], [0, 1], [0], g["k1"], g["b"])
+    assert avgdl == pytest.approx(11 / 6, abs=1e-15)
+    assert df[0] == 2 and df[5] == 1 and df[2] == 1
+    idf = np.log(1 + (6 - 2 + 0.5) / (2 + 0.5))
+    L0 = 0.25 + 0.75 * 2 / (11 / 6)
+    L5 = 0.25 + 0.75 * 1 / (11 / 6)
+    np.testing.assert_allclose(M[0], [idf * 2.2 / (1 + 1.2 * L0), 0, 0, 0, 0,
+                                      idf * 2.2 / (1 + 1.2 * L5)], rtol=1e-14)
+
+
+def test_search_two_is_the_search_of_the_stacked_index():
+    w = workloads.config(1, n=500, batch=7)
+    Ek, Em = w.E_data[:320], w.E_data[320:]
+    ids, src, sc = oracle.search_two(Ek, Em, w.Q_data, 12)
+    f_ids, f_sc = oracle.search(w.E_data, w.Q_data, 12)
+    np.testing.assert_array_equal(np.where(src == 1, ids + 320, ids), f_ids)
+    np.testing.assert_array_equal(sc, f_sc)
+    # a memory index equal to the knowledge index: every score appears twice,
+    # the knowledge copy first
+    ids2, src2, sc2 = oracle.search_two(Ek, Ek, w.Q_data, 6)
+    assert (ids2[:, 0::2] == ids2[:, 1::2]).all()
+    assert (src2[:, 0::2] == 0).all() and (src2[:, 1::2] == 1).all()
+
+
 # ------------------------------------------------------------------ upsert
 
 def test_upsert_last_duplicate_wins_and_matches_rebuild():
