@@ -200,6 +200,41 @@ OPRAG_API int oprag_embed_pool(const void *hidden, int32_t hidden_dtype, int32_t
                                int32_t out_dtype, void *stream);
 
 /*
+ * Appends m rows as chunks n, n + 1, ... (Op_upsert inserting, Sec. 3.2;
+ * Sec. 4.4: the memory index grows by upserts).  The device buffer grows by
+ * doubling (a reallocation: earlier oprag_index_data pointers become
+ * invalid).  *first_id (optional) receives the id of the first new chunk.
+ * With a sparse side attached, the new chunks hold no terms (see
+ * oprag_index_update_sparse) and the BM25 statistics are rebuilt for the new
+ * chunk count.  rows / rows_dtype / rows_on_device as oprag_upsert.
+ * Synchronous when the buffer grows or a sparse side is attached.
+ */
+OPRAG_API int oprag_append(oprag_index *idx, const void *rows, int64_t m, int32_t rows_dtype,
+                           int32_t rows_on_device, int64_t *first_id, void *stream);
+
+/*
+ * Replaces the token bags of chunks ids[0..m) (host, each in [0, n); a later
+ * duplicate wins) by the host CSR bags bag_indptr[m + 1] / bag_terms, and
+ * rebuilds df, avgdl and every BM25 weight so that the lexical scores stay
+ * exact over the updated corpus (the lexical half of Op_upsert, Sec. 3.2).
+ * Synchronous.  OPRAG_ERR_NOT_READY without a sparse side.
+ */
+OPRAG_API int oprag_index_update_sparse(oprag_index *idx, const int64_t *ids, int64_t m,
+                                        const int32_t *bag_indptr, const int32_t *bag_terms);
+
+/*
+ * Dense top-k over a knowledge index and a memory index together (Sec. 4.4:
+ * both indices are searched the same way; one ranked result).  Same dim and
+ * dtype on the same device.  out_ids: chunk id within its index; out_src: 0 =
+ * knowledge, 1 = memory (device, q x k each, out_scores as oprag_search).
+ * Order: score descending, then knowledge before memory, then chunk id.
+ * k <= n_knowledge + n_memory.  Asynchronous on `stream`.
+ */
+OPRAG_API int oprag_search_two(oprag_index *knowledge, oprag_index *memory, const void *queries,
+                               int32_t q, int32_t k, int64_t *out_ids, int32_t *out_src,
+                               float *out_scores, void *stream);
+
+/*
  * Waits for the index's pending work and reports whether a kernel of it gave
  * up a bounded wait since the last check (OPRAG_ERR_DEVICE; the flag is then
  * cleared) or a CUDA error occurred (OPRAG_ERR_CUDA).

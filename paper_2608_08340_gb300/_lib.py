@@ -51,6 +51,9 @@ SIGNATURES = {
     "oprag_index_set_option": (_I32, [_P, _I32, _I32]),
     "oprag_hybrid_search_dense_first": (_I32, [_P, _P, _I32, _P, _P, _F, _I32, _I32, _P, _P, _P]),
     "oprag_embed_pool": (_I32, [_P, _I32, _I32, _I32, _I32, _P, _P, _I32, _P]),
+    "oprag_append": (_I32, [_P, _P, _I64, _I32, _I32, _P, _P]),
+    "oprag_index_update_sparse": (_I32, [_P, _P, _I64, _P, _P]),
+    "oprag_search_two": (_I32, [_P, _P, _P, _I32, _I32, _P, _P, _P, _P]),
     "oprag_index_last_path": (_I32, [_P]),
     "oprag_index_last_launch": (_I32, [_P, ctypes.POINTER(_I32), ctypes.POINTER(_I32),
                                        ctypes.POINTER(_I32)]),

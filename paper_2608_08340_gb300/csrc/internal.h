@@ -109,6 +109,14 @@ inline __host__ __device__ int level_rank(int k, int i) {
 cudaError_t launch_merge(const ListSet& ls, int q, int k, int64_t* out_ids, float* out_scores,
                          cudaStream_t st, float* kth_out = nullptr, float* levels_out = nullptr);
 
+// Two ranked lists per query (a: q x ka, b: q x kb, each sorted score
+// descending then id ascending) into the top-k of both, score descending,
+// then list a before list b, then id; out_src: 0 = a, 1 = b.
+cudaError_t launch_merge_two(int q, const int64_t* a_ids, const float* a_sc, int ka,
+                             const int64_t* b_ids, const float* b_sc, int kb, int k,
+                             int64_t* out_ids, int32_t* out_src, float* out_scores,
+                             cudaStream_t st);
+
 // --- BM25 matrix pass (lexical part of the hybrid search).
 // Per-posting weight w(t, d) = idf * tf (k1+1) / (tf + k1 (1 - b + b |d| / avgdl)).
 // Terms held by more than half of the chunks are stored as dense rows of

@@ -210,6 +210,58 @@ cudaError_t launch_warp_per_query(Kern kern, int warps, const ListSet& ls, int q
 
 }  // namespace
 
+namespace {
+
+// One thread per query: a two-way merge of the queries' ranked lists.
+__global__ void merge_two_kernel(int q, const int64_t* __restrict__ a_ids,
+                                 const float* __restrict__ a_sc, int ka,
+                                 const int64_t* __restrict__ b_ids,
+                                 const float* __restrict__ b_sc, int kb, int k,
+                                 int64_t* __restrict__ out_ids, int32_t* __restrict__ out_src,
+                                 float* __restrict__ out_scores) {
+  const int qi = blockIdx.x * blockDim.x + threadIdx.x;
+  if (qi >= q) return;
+  const int64_t* ai = a_ids + static_cast<int64_t>(qi) * ka;
+  const float* as = a_sc + static_cast<int64_t>(qi) * ka;
+  const int64_t* bi = b_ids + static_cast<int64_t>(qi) * kb;
+  const float* bs = b_sc + static_cast<int64_t>(qi) * kb;
+  int i = 0, j = 0;
+  for (int r = 0; r < k; ++r) {
+    const bool a_ok = i < ka && ai[i] >= 0;
+    const bool b_ok = j < kb && bi[j] >= 0;
+    // At equal scores list a (the knowledge index) comes first.
+    const bool take_a = a_ok && (!b_ok || !(bs[j] > as[i]));
+    const int64_t o = static_cast<int64_t>(qi) * k + r;
+    if (take_a) {
+      out_ids[o] = ai[i];
+      out_scores[o] = as[i];
+      out_src[o] = 0;
+      ++i;
+    } else if (b_ok) {
+      out_ids[o] = bi[j];
+      out_scores[o] = bs[j];
+      out_src[o] = 1;
+      ++j;
+    } else {
+      out_ids[o] = -1;
+      out_scores[o] = -INFINITY;
+      out_src[o] = -1;
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_merge_two(int q, const int64_t* a_ids, const float* a_sc, int ka,
+                             const int64_t* b_ids, const float* b_sc, int kb, int k,
+                             int64_t* out_ids, int32_t* out_src, float* out_scores,
+                             cudaStream_t st) {
+  if (q <= 0) return cudaSuccess;
+  merge_two_kernel<<<(q + 127) / 128, 128, 0, st>>>(q, a_ids, a_sc, ka, b_ids, b_sc, kb, k,
+                                                    out_ids, out_src, out_scores);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_merge(const ListSet& ls, int q, int k, int64_t* out_ids, float* out_scores,
                          cudaStream_t st, float* kth_out, float* levels_out) {
   if (q <= 0) return cudaSuccess;

@@ -66,6 +66,7 @@ struct oprag_index {
   int device = 0;
   int num_sms = 1;
   int64_t n = 0;
+  int64_t cap = 0;             // rows allocated for emb (appends double it)
   int d = 0;
   int dtype = OPRAG_BF16;
   void* emb = nullptr;
@@ -83,6 +84,10 @@ struct oprag_index {
 
   bool has_sparse = false;
   int vocab = 0;
+  // Host copy of the token bags (CSR) and BM25 parameters: the device side is
+  // rebuilt from them when bags are replaced or chunks appended.
+  std::vector<int32_t> bag_ptr, bag_terms;
+  double bm_k1 = 1.2, bm_b = 0.75;
   int64_t nnz = 0;
   int64_t* post_ptr = nullptr;
   int2* post = nullptr;
@@ -335,6 +340,7 @@ int oprag_index_create(oprag_index** out, const void* emb, int64_t n, int32_t d,
   }
   cudaDeviceGetAttribute(&idx->num_sms, cudaDevAttrMultiProcessorCount, idx->device);
   idx->n = n;
+  idx->cap = n;
   idx->d = d;
   idx->dtype = dtype;
   const size_t count = static_cast<size_t>(n) * d;
@@ -518,6 +524,104 @@ int oprag_upsert(oprag_index* idx, const int64_t* ids, const void* rows, int64_t
   return end_call(idx, st);
 }
 
+int rebuild_sparse(oprag_index* idx);
+
+int oprag_append(oprag_index* idx, const void* rows, int64_t m, int32_t rows_dtype,
+                 int32_t rows_on_device, int64_t* first_id, void* stream) {
+  if (!idx) return fail(OPRAG_ERR_INVALID_ARG, "index is NULL");
+  if (m < 0) return fail(OPRAG_ERR_INVALID_ARG, "m < 0");
+  if (first_id) *first_id = idx->n;
+  if (m == 0) return ok();
+  if (!rows) return fail(OPRAG_ERR_INVALID_ARG, "NULL rows");
+  if (rows_dtype != OPRAG_F32 && rows_dtype != OPRAG_BF16)
+    return fail(OPRAG_ERR_INVALID_ARG, "unknown rows dtype");
+  if (idx->dtype == OPRAG_F32 && rows_dtype == OPRAG_BF16)
+    return fail(OPRAG_ERR_INVALID_ARG, "bf16 rows into an f32 index are not supported");
+  if (idx->n + m > (int64_t(1) << 31))
+    return fail(OPRAG_ERR_INVALID_ARG, "an index holds at most 2^31 chunks");
+  DeviceGuard g(idx->device);
+  const int64_t n0 = idx->n;
+  if (n0 + m > idx->cap) {
+    // Capacity doubling: a new allocation, the rows so far copied over.
+    cudaError_t e = idx->drain();
+    if (e != cudaSuccess) return cuda_fail(e, "waiting for pending work");
+    const int64_t cap = std::max<int64_t>(n0 + m, 2 * idx->cap);
+    const size_t row_bytes = static_cast<size_t>(idx->d) * elem_size(idx->dtype);
+    void* grown = nullptr;
+    if (cudaMalloc(&grown, static_cast<size_t>(cap) * row_bytes) != cudaSuccess) {
+      cudaGetLastError();
+      return fail(OPRAG_ERR_OOM, "cannot grow the index to %lld rows", (long long)cap);
+    }
+    e = cudaMemcpy(grown, idx->emb, static_cast<size_t>(n0) * row_bytes, cudaMemcpyDeviceToDevice);
+    if (e != cudaSuccess) {
+      cudaFree(grown);
+      return cuda_fail(e, "copying the index");
+    }
+    cudaFree(idx->emb);
+    idx->emb = grown;
+    idx->cap = cap;
+  }
+  idx->n = n0 + m;
+  std::vector<int64_t> ids(static_cast<size_t>(m));
+  for (int64_t i = 0; i < m; ++i) ids[i] = n0 + i;
+  int rc = oprag_upsert(idx, ids.data(), rows, m, rows_dtype, rows_on_device, stream);
+  if (rc) {
+    idx->n = n0;
+    return rc;
+  }
+  if (idx->has_sparse) {
+    // The new chunks hold no terms yet (oprag_index_update_sparse gives them
+    // bags); N and avgdl change, so every BM25 weight is rebuilt.
+    cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "appending rows");
+    idx->bag_ptr.resize(static_cast<size_t>(idx->n) + 1, idx->bag_ptr.back());
+    return rebuild_sparse(idx);
+  }
+  return ok();
+}
+
+int oprag_search_two(oprag_index* knowledge, oprag_index* memory, const void* queries, int32_t q,
+                     int32_t k, int64_t* out_ids, int32_t* out_src, float* out_scores,
+                     void* stream) {
+  if (!knowledge || !memory) return fail(OPRAG_ERR_INVALID_ARG, "index is NULL");
+  if (knowledge->d != memory->d || knowledge->dtype != memory->dtype ||
+      knowledge->device != memory->device)
+    return fail(OPRAG_ERR_INVALID_ARG, "the two indices differ in dim, dtype or device");
+  if (!out_src) return fail(OPRAG_ERR_INVALID_ARG, "NULL out_src");
+  if (k < 1 || k > OPRAG_K_MAX || k > knowledge->n + memory->n)
+    return fail(OPRAG_ERR_INVALID_ARG, "k = %d outside [1, min(%d, n_knowledge + n_memory)]", k,
+                OPRAG_K_MAX);
+  if (q < 0) return fail(OPRAG_ERR_INVALID_ARG, "q < 0");
+  if (q == 0) return ok();
+  if (!queries || !out_ids || !out_scores) return fail(OPRAG_ERR_INVALID_ARG, "NULL argument");
+  const int ka = static_cast<int>(std::min<int64_t>(k, knowledge->n));
+  const int kb = static_cast<int>(std::min<int64_t>(k, memory->n));
+  DeviceGuard g(knowledge->device);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // Each index's top-k into its own candidate buffer, then one merge.
+  int rc;
+  if ((rc = knowledge->ensure(&knowledge->cand, &knowledge->cand_bytes,
+                              static_cast<size_t>(q) * ka * 12, "two-index results")))
+    return rc;
+  if ((rc = memory->ensure(&memory->cand, &memory->cand_bytes,
+                           static_cast<size_t>(q) * kb * 12, "two-index results")))
+    return rc;
+  if ((rc = begin_call(knowledge, st))) return rc;
+  if ((rc = begin_call(memory, st))) return rc;
+  int64_t* a_ids = static_cast<int64_t*>(knowledge->cand);
+  float* a_sc = reinterpret_cast<float*>(a_ids + static_cast<size_t>(q) * ka);
+  int64_t* b_ids = static_cast<int64_t*>(memory->cand);
+  float* b_sc = reinterpret_cast<float*>(b_ids + static_cast<size_t>(q) * kb);
+  const Fusion none{nullptr, 0, nullptr, 0.f};
+  if ((rc = run_search(knowledge, queries, q, ka, none, a_ids, a_sc, st))) return rc;
+  if ((rc = run_search(memory, queries, q, kb, none, b_ids, b_sc, st))) return rc;
+  cudaError_t e = launch_merge_two(q, a_ids, a_sc, ka, b_ids, b_sc, kb, k, out_ids, out_src,
+                                   out_scores, st);
+  if (e != cudaSuccess) return cuda_fail(e, "two-index merge");
+  if ((rc = end_call(memory, st))) return rc;
+  return end_call(knowledge, st);
+}
+
 int oprag_search(oprag_index* idx, const void* queries, int32_t q, int32_t k, int64_t* out_ids,
                  float* out_scores, void* stream) {
   int rc = check_search_args(idx, queries, q, k, out_ids, out_scores);
@@ -564,22 +668,17 @@ int oprag_search_host(oprag_index* idx, const void* queries, int32_t q, int32_t 
   return oprag_index_check(idx);
 }
 
-int oprag_index_set_sparse(oprag_index* idx, const int32_t* doc_indptr, const int32_t* doc_terms,
-                           int32_t vocab, float k1, float b) {
-  if (!idx || !doc_indptr) return fail(OPRAG_ERR_INVALID_ARG, "NULL argument");
-  if (vocab < 1) return fail(OPRAG_ERR_INVALID_ARG, "vocab = %d", vocab);
-  if (!(k1 >= 0.f) || !(b >= 0.f && b <= 1.f))
-    return fail(OPRAG_ERR_INVALID_ARG, "need k1 >= 0 and 0 <= b <= 1");
+// Builds the device side of BM25 (per-posting weights, dense rows of the
+// commonest terms, postings) from the index's host copy of the token bags,
+// in fp64 on the host.  Called whenever the bags or the chunk count change,
+// so that df, avgdl and every weight follow the current corpus.
+int rebuild_sparse(oprag_index* idx) {
   const int64_t n = idx->n;
-  if (doc_indptr[0] != 0) return fail(OPRAG_ERR_INVALID_ARG, "doc_indptr[0] != 0");
-  for (int64_t i = 0; i < n; ++i)
-    if (doc_indptr[i + 1] < doc_indptr[i])
-      return fail(OPRAG_ERR_INVALID_ARG, "doc_indptr decreases at %lld", (long long)i);
+  const int vocab = idx->vocab;
+  const double k1 = idx->bm_k1, b = idx->bm_b;
+  const int32_t* doc_indptr = idx->bag_ptr.data();
+  const int32_t* doc_terms = idx->bag_terms.data();
   const int64_t total = doc_indptr[n];
-  if (total > 0 && !doc_terms) return fail(OPRAG_ERR_INVALID_ARG, "doc_terms is NULL");
-  for (int64_t p = 0; p < total; ++p)
-    if (doc_terms[p] < 0 || doc_terms[p] >= vocab)
-      return fail(OPRAG_ERR_INVALID_ARG, "term id %d outside [0, %d)", doc_terms[p], vocab);
 
   // Term frequencies per chunk, document frequencies, average length.
   std::vector<int64_t> df(vocab, 0);
@@ -601,7 +700,7 @@ int oprag_index_set_sparse(oprag_index* idx, const int32_t* doc_indptr, const in
       i = j;
     }
   }
-  const double avgdl = static_cast<double>(total) / static_cast<double>(n);
+  const double avgdl = n > 0 ? static_cast<double>(total) / static_cast<double>(n) : 0.0;
   // Terms in more than half of the chunks become dense rows; the others
   // keep postings grouped by term, chunks ascending inside a term.
   std::vector<int32_t> slot(vocab, -1);
@@ -637,6 +736,7 @@ int oprag_index_set_sparse(oprag_index* idx, const int32_t* doc_indptr, const in
   cudaError_t e = idx->drain();
   if (e != cudaSuccess) return cuda_fail(e, "waiting for pending work");
   idx->free_sparse();
+  idx->has_sparse = false;
   if (cudaMalloc(&idx->post_ptr, ptr.size() * sizeof(int64_t)) != cudaSuccess ||
       cudaMalloc(&idx->post, std::max<int64_t>(nnz, 1) * sizeof(int2)) != cudaSuccess ||
       cudaMalloc(&idx->dense_slot, slot.size() * sizeof(int32_t)) != cudaSuccess ||
@@ -656,11 +756,75 @@ int oprag_index_set_sparse(oprag_index* idx, const int32_t* doc_indptr, const in
     idx->free_sparse();
     return cuda_fail(e, "uploading postings");
   }
-  idx->vocab = vocab;
   idx->nnz = nnz;
   idx->dense_ld = dld;
   idx->has_sparse = true;
   return ok();
+}
+
+// Term ids of bags must lie in [0, vocab).
+int check_bags(const int32_t* indptr, const int32_t* terms, int64_t count, int vocab) {
+  if (indptr[0] != 0) return fail(OPRAG_ERR_INVALID_ARG, "bag indptr[0] != 0");
+  for (int64_t i = 0; i < count; ++i)
+    if (indptr[i + 1] < indptr[i])
+      return fail(OPRAG_ERR_INVALID_ARG, "bag indptr decreases at %lld", (long long)i);
+  const int64_t total = indptr[count];
+  if (total > 0 && !terms) return fail(OPRAG_ERR_INVALID_ARG, "bag terms is NULL");
+  for (int64_t p = 0; p < total; ++p)
+    if (terms[p] < 0 || terms[p] >= vocab)
+      return fail(OPRAG_ERR_INVALID_ARG, "term id %d outside [0, %d)", terms[p], vocab);
+  return OPRAG_OK;
+}
+
+int oprag_index_set_sparse(oprag_index* idx, const int32_t* doc_indptr, const int32_t* doc_terms,
+                           int32_t vocab, float k1, float b) {
+  if (!idx || !doc_indptr) return fail(OPRAG_ERR_INVALID_ARG, "NULL argument");
+  if (vocab < 1) return fail(OPRAG_ERR_INVALID_ARG, "vocab = %d", vocab);
+  if (!(k1 >= 0.f) || !(b >= 0.f && b <= 1.f))
+    return fail(OPRAG_ERR_INVALID_ARG, "need k1 >= 0 and 0 <= b <= 1");
+  int rc = check_bags(doc_indptr, doc_terms, idx->n, vocab);
+  if (rc) return rc;
+  const int64_t total = doc_indptr[idx->n];
+  idx->bag_ptr.assign(doc_indptr, doc_indptr + idx->n + 1);
+  idx->bag_terms.assign(doc_terms, doc_terms + total);
+  idx->vocab = vocab;
+  idx->bm_k1 = k1;
+  idx->bm_b = b;
+  return rebuild_sparse(idx);
+}
+
+int oprag_index_update_sparse(oprag_index* idx, const int64_t* ids, int64_t m,
+                              const int32_t* bag_indptr, const int32_t* bag_terms) {
+  if (!idx) return fail(OPRAG_ERR_INVALID_ARG, "index is NULL");
+  if (!idx->has_sparse) return fail(OPRAG_ERR_NOT_READY, "no sparse side: call oprag_index_set_sparse");
+  if (m < 0) return fail(OPRAG_ERR_INVALID_ARG, "m < 0");
+  if (m == 0) return ok();
+  if (!ids || !bag_indptr) return fail(OPRAG_ERR_INVALID_ARG, "NULL argument");
+  for (int64_t i = 0; i < m; ++i)
+    if (ids[i] < 0 || ids[i] >= idx->n)
+      return fail(OPRAG_ERR_RANGE, "ids[%lld] = %lld outside [0, %lld)", (long long)i,
+                  (long long)ids[i], (long long)idx->n);
+  int rc = check_bags(bag_indptr, bag_terms, m, idx->vocab);
+  if (rc) return rc;
+  // New bags: the last occurrence of a repeated id wins.
+  std::vector<int64_t> which(static_cast<size_t>(idx->n), -1);
+  for (int64_t i = 0; i < m; ++i) which[ids[i]] = i;
+  std::vector<int32_t> ptr(static_cast<size_t>(idx->n) + 1, 0), terms;
+  terms.reserve(idx->bag_terms.size());
+  for (int64_t dd = 0; dd < idx->n; ++dd) {
+    const int64_t w = which[dd];
+    if (w < 0)
+      terms.insert(terms.end(), idx->bag_terms.begin() + idx->bag_ptr[dd],
+                   idx->bag_terms.begin() + idx->bag_ptr[dd + 1]);
+    else
+      terms.insert(terms.end(), bag_terms + bag_indptr[w], bag_terms + bag_indptr[w + 1]);
+    if (terms.size() > static_cast<size_t>(INT32_MAX))
+      return fail(OPRAG_ERR_INVALID_ARG, "token bags exceed 2^31 terms");
+    ptr[dd + 1] = static_cast<int32_t>(terms.size());
+  }
+  idx->bag_ptr.swap(ptr);
+  idx->bag_terms.swap(terms);
+  return rebuild_sparse(idx);
 }
 
 int oprag_hybrid_search(oprag_index* idx, const void* queries, int32_t q, const int32_t* q_indptr,

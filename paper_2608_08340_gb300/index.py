@@ -166,6 +166,29 @@ class Index:
         check(self._lib.oprag_upsert(self._h, ids_np.ctypes.data, _ptr(rows), ids_np.shape[0],
                                      _DT[rows.dtype], int(rows.is_cuda), _stream_ptr(stream)))
 
+    def append(self, rows: torch.Tensor, stream=None) -> int:
+        """Appends rows as chunks n, n + 1, ...; returns the first new id."""
+        if rows.dim() != 2 or rows.shape[1] != self.d or rows.dtype not in _DT:
+            raise ValueError(f"rows must be (m, {self.d}) float32 or bfloat16")
+        rows = rows.contiguous()
+        first = ctypes.c_int64()
+        check(self._lib.oprag_append(self._h, _ptr(rows), int(rows.shape[0]), _DT[rows.dtype],
+                                     int(rows.is_cuda), ctypes.byref(first), _stream_ptr(stream)))
+        self.n += int(rows.shape[0])
+        return int(first.value)
+
+    def update_sparse(self, ids, bag_indptr, bag_terms) -> None:
+        """Replaces the token bags of chunks ids (host CSR bags, later duplicates win)."""
+        ids_np = np.ascontiguousarray(ids, dtype=np.int64)
+        ip = np.ascontiguousarray(bag_indptr, dtype=np.int32)
+        tm = np.ascontiguousarray(bag_terms, dtype=np.int32)
+        if ip.shape[0] != ids_np.shape[0] + 1:
+            raise ValueError("bag_indptr must have len(ids) + 1 entries")
+        if tm.size == 0:
+            tm = np.zeros(1, np.int32)
+        check(self._lib.oprag_index_update_sparse(self._h, ids_np.ctypes.data, ids_np.shape[0],
+                                                  ip.ctypes.data, tm.ctypes.data))
+
     # -- misc
     def rows(self, first: int = 0, count: int | None = None) -> torch.Tensor:
         count = self.n - first if count is None else count
@@ -237,4 +260,17 @@ def embed_pool(hidden: torch.Tensor, mask: torch.Tensor, out_dtype: torch.dtype 
     check(lib.oprag_embed_pool(_ptr(hidden), _DT[hidden.dtype], b, t, d, _ptr(m), _ptr(out),
                                _DT[out_dtype], _stream_ptr(stream)))
     return out
+
+
+def search_two(knowledge: Index, memory: Index, queries: torch.Tensor, k: int, stream=None):
+    """Dense top-k over a knowledge and a memory index: (ids, src, scores);
+    src 0 = knowledge, 1 = memory; ids are chunk ids within their index."""
+    queries = knowledge._queries(queries)
+    q = int(queries.shape[0])
+    ids = torch.empty((q, k), dtype=torch.int64, device=queries.device)
+    src = torch.empty((q, k), dtype=torch.int32, device=queries.device)
+    scores = torch.empty((q, k), dtype=torch.float32, device=queries.device)
+    check(knowledge._lib.oprag_search_two(knowledge._h, memory._h, _ptr(queries), q, k, _ptr(ids),
+                                          _ptr(src), _ptr(scores), _stream_ptr(stream)))
+    return ids, src, scores
 
