@@ -76,6 +76,9 @@ def parse():
     p.add_argument("--embed-tail", action="store_true",
                    help="time the embedding tail instead (masked mean pool + L2 normalise of "
                         "256 x 512 x 4096 bf16 hidden states, the Llama3-8B hidden size)")
+    p.add_argument("--index-ops", action="store_true",
+                   help="time the index updates instead: append of 4096 rows, replacement of "
+                        "4096 token bags (BM25 rebuilt), search over a knowledge + memory index")
     p.add_argument("--dense-first", type=int, default=0, metavar="N",
                    help="config 3 only: dense top-N, then the lexical rerank of those N "
                         "candidates (dense-first hybrid) instead of the full hybrid")
@@ -605,10 +608,82 @@ def run_embed_tail(args):
         "gpu_launches": args.steps}))
 
 
+def run_index_ops(args):
+    """Index updates (Sec. 3.2 Op_upsert, Sec. 4.4 memory index): append
+    (rows/s), token-bag replacement (wall time of the rebuild), and the
+    knowledge + memory search against the knowledge search alone."""
+    import torch
+    from paper_2608_08340_gb300.index import Index, search_two
+
+    torch.cuda.set_device(0)
+    w = workloads.config(3, batch=256)
+    dev = torch.device("cuda", 0)
+    to_dev = lambda a: torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).to(dev)
+    out = {}
+    # append: a 32768-chunk index grows by 4096 rows per step
+    rows = to_dev(workloads.upsert_batch(w.n, w.d, 4096, 1, "bf16")[1])
+    idx = Index(to_dev(w.E_data))
+    idx.append(rows)                             # first growth (doubling) outside the timing
+    times = []
+    for _ in range(args.steps):
+        a = torch.cuda.Event(enable_timing=True)
+        e = torch.cuda.Event(enable_timing=True)
+        a.record()
+        idx.append(rows)
+        e.record()
+        torch.cuda.synchronize()
+        times.append(a.elapsed_time(e))
+    out["append_4096_rows_ms"] = statistics.median(times)
+    out["append_rows_per_s"] = 4096 / (statistics.median(times) * 1e-3)
+    out["index_rows_after"] = idx.n
+    idx.close()
+    # token bags: 4096 chunks get new bags, BM25 rebuilt on the host and uploaded
+    idx = Index(to_dev(w.E_data))
+    idx.set_sparse(w.doc_indptr, w.doc_terms, w.vocab, w.k1, w.b)
+    rng = np.random.default_rng(6000)
+    ids = rng.choice(w.n, 4096, replace=False)
+    bip = (w.doc_indptr[ids + 1] - w.doc_indptr[ids]).cumsum()
+    bip = np.concatenate([[0], bip]).astype(np.int32)
+    btm = rng.choice(w.doc_terms, int(bip[-1])).astype(np.int32)
+    times = []
+    for _ in range(max(3, args.steps // 10)):
+        t0 = time.perf_counter()
+        idx.update_sparse(ids, bip, btm)
+        times.append((time.perf_counter() - t0) * 1e3)
+    out["update_4096_bags_ms"] = statistics.median(times)
+    idx.close()
+    # knowledge (32768) + memory (8192) search of 256 queries against knowledge alone
+    kn = Index(to_dev(w.E_data))
+    mem = Index(to_dev(workloads.config(1, n=8192, batch=1).E_data))
+    Q = to_dev(workloads.config(1, batch=256).Q_data)
+    for label, fn in (("search_knowledge_ms", lambda: kn.search(Q, w.k)),
+                      ("search_two_ms", lambda: search_two(kn, mem, Q, w.k))):
+        for _ in range(args.warmup):
+            fn()
+        marks = []
+        for _ in range(args.steps):
+            a = torch.cuda.Event(enable_timing=True)
+            e = torch.cuda.Event(enable_timing=True)
+            a.record()
+            fn()
+            e.record()
+            marks.append((a, e))
+        torch.cuda.synchronize()
+        out[label] = statistics.median(a.elapsed_time(e) for a, e in marks)
+    print(json.dumps({"metric": "index update timings", "unit": "ms", "n_gpus": 1,
+                      "steps": args.steps, "warmup": args.warmup, "data": "synthetic",
+                      "config": {"workload": "32768 x 768 bf16 knowledge index, 8192-row memory "
+                                             "index, 256 queries, 4096-row updates"},
+                      "results": out}))
+
+
 def main():
     args = parse()
     if args.embed_tail and args.impl == "ours":
         run_embed_tail(args)
+        return
+    if args.index_ops and args.impl == "ours":
+        run_index_ops(args)
         return
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
