@@ -260,6 +260,15 @@ OPRAG_API int oprag_index_set_option(oprag_index *idx, int32_t option, int32_t v
  * then cleared). */
 #define OPRAG_OPT_BOUND_TAG 5
 
+/* OPRAG_OPT_GRAPH: 1 makes oprag_search capture its launches into a CUDA graph
+ * when it is called again with the same queries / outputs pointers, q, k and
+ * stream and the index has not changed (no growth, append or option change
+ * since), and replay that graph on later identical calls (one launch instead
+ * of several).  The stream must not be the legacy default stream; calls on
+ * other streams keep their ordering through the index's completion event.
+ * 0 (default) off. */
+#define OPRAG_OPT_GRAPH 6
+
 /* OPRAG_OPT_TIMING: 1 makes every later search record CUDA events, on the
  * call's stream, around its lexical (BM25) kernel, its main search kernel and
  * its merge kernel; oprag_index_last_timing() reads them.  0 (default) off. */

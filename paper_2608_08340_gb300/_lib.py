@@ -17,6 +17,7 @@ OPRAG_OPT_BLOCK_N = 2
 OPRAG_OPT_TIMING = 3
 OPRAG_OPT_PAIR = 4
 OPRAG_OPT_BOUND_TAG = 5
+OPRAG_OPT_GRAPH = 6
 
 ERRORS = {
     0: "OK",

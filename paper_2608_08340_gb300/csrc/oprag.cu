@@ -98,6 +98,21 @@ struct oprag_index {
   int opt_path = 0;
   int opt_block_n = 0;
   int opt_pair = 0;
+  // Replay of a captured dense search (OPRAG_OPT_GRAPH): the launches of the
+  // previous search with the same pointers, sizes, stream and index state.
+  int opt_graph = 0;
+  uint64_t state_version = 0;  // bumped whenever a buffer moves or an option changes
+  bool capturing = false;
+  struct {
+    bool seen = false;
+    const void* queries = nullptr;
+    int q = 0, k = 0;
+    int64_t* ids = nullptr;
+    float* scores = nullptr;
+    cudaStream_t st = nullptr;
+    uint64_t version = 0;
+    cudaGraphExec_t exec = nullptr;
+  } gcache;
   // Per-query k-th score bounds shared by the lists of one search, tagged
   // with a per-launch generation (zeroed memory holds no valid entry).
   uint64_t* qfloor = nullptr;
@@ -121,6 +136,7 @@ struct oprag_index {
   // an earlier call enqueued, so the whole device is drained first.
   int ensure(void** buf, size_t* cur, size_t need, const char* what) {
     if (need <= *cur) return OPRAG_OK;
+    ++state_version;
     cudaError_t e = cudaDeviceSynchronize();
     if (e != cudaSuccess) return cuda_fail(e, "waiting for pending work");
     if (*buf) cudaFree(*buf);
@@ -185,6 +201,12 @@ int shared_floors(oprag_index* idx, int q, cudaStream_t st, uint64_t** qf, uint3
                          "shared k-th score bounds");
     if (rc) return rc;
     cudaError_t e = cudaMemsetAsync(idx->qfloor, 0, idx->qfloor_bytes, st);
+    if (e != cudaSuccess) return cuda_fail(e, "clearing shared bounds");
+  }
+  if (idx->capturing) {
+    // A captured search is replayed with the same tag: clear its entries in
+    // every replay instead.
+    cudaError_t e = cudaMemsetAsync(idx->qfloor, 0, need, st);
     if (e != cudaSuccess) return cuda_fail(e, "clearing shared bounds");
   }
   if (++idx->gen == 0) {            // tags wrapped: old entries could read as current
@@ -401,6 +423,7 @@ void oprag_index_destroy(oprag_index* idx) {
   idx->drain();
   if (idx->emb) cudaFree(idx->emb);
   if (idx->dev_err) cudaFree(idx->dev_err);
+  if (idx->gcache.exec) cudaGraphExecDestroy(idx->gcache.exec);
   if (idx->scratch) cudaFree(idx->scratch);
   if (idx->qfloor) cudaFree(idx->qfloor);
   if (idx->lex) cudaFree(idx->lex);
@@ -562,6 +585,7 @@ int oprag_append(oprag_index* idx, const void* rows, int64_t m, int32_t rows_dty
     idx->cap = cap;
   }
   idx->n = n0 + m;
+  ++idx->state_version;
   std::vector<int64_t> ids(static_cast<size_t>(m));
   for (int64_t i = 0; i < m; ++i) ids[i] = n0 + i;
   int rc = oprag_upsert(idx, ids.data(), rows, m, rows_dtype, rows_on_device, stream);
@@ -632,6 +656,55 @@ int oprag_search(oprag_index* idx, const void* queries, int32_t q, int32_t k, in
   if ((rc = begin_call(idx, st))) return rc;
   const Fusion none{nullptr, 0, nullptr, 0.f};
   idx->timed_lex = false;
+  // Graph mode: a search repeated with the same pointers, sizes, stream and
+  // index state is captured once (on its second call) and then replayed
+  // with one graph launch.  Not on the legacy default stream (no capture).
+  auto& c = idx->gcache;
+  if (idx->opt_graph && st != nullptr && !idx->timing) {
+    const bool same = c.seen && c.queries == queries && c.q == q && c.k == k &&
+                      c.ids == out_ids && c.scores == out_scores && c.st == st &&
+                      c.version == idx->state_version;
+    if (same && c.exec) {
+      cudaError_t e = cudaGraphLaunch(c.exec, st);
+      if (e != cudaSuccess) return cuda_fail(e, "graph launch");
+      return end_call(idx, st);
+    }
+    if (same) {
+      cudaError_t e = cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal);
+      if (e == cudaSuccess) {
+        idx->capturing = true;
+        rc = run_search(idx, queries, q, k, none, out_ids, out_scores, st);
+        idx->capturing = false;
+        cudaGraph_t graph = nullptr;
+        e = cudaStreamEndCapture(st, &graph);
+        cudaGraphExec_t exec = nullptr;
+        if (rc == OPRAG_OK && e == cudaSuccess && graph)
+          e = cudaGraphInstantiate(&exec, graph, 0);
+        if (graph) cudaGraphDestroy(graph);
+        if (rc == OPRAG_OK && e == cudaSuccess && exec) {
+          c.exec = exec;
+          if ((e = cudaGraphLaunch(exec, st)) != cudaSuccess) return cuda_fail(e, "graph launch");
+          return end_call(idx, st);
+        }
+        if (exec) cudaGraphExecDestroy(exec);
+        cudaGetLastError();
+      } else {
+        cudaGetLastError();
+      }
+      c.seen = false;            // this search does not capture: launch it directly
+    } else {
+      if (c.exec) cudaGraphExecDestroy(c.exec);
+      c.exec = nullptr;
+      c.seen = true;
+      c.queries = queries;
+      c.q = q;
+      c.k = k;
+      c.ids = out_ids;
+      c.scores = out_scores;
+      c.st = st;
+      c.version = idx->state_version;
+    }
+  }
   if ((rc = run_search(idx, queries, q, k, none, out_ids, out_scores, st))) return rc;
   return end_call(idx, st);
 }
@@ -938,6 +1011,12 @@ int oprag_index_check(oprag_index* idx) {
 
 int oprag_index_set_option(oprag_index* idx, int32_t option, int32_t value) {
   if (!idx) return fail(OPRAG_ERR_INVALID_ARG, "index is NULL");
+  ++idx->state_version;
+  if (option == OPRAG_OPT_GRAPH) {
+    if (value < 0 || value > 1) return fail(OPRAG_ERR_INVALID_ARG, "graph mode %d", value);
+    idx->opt_graph = value;
+    return ok();
+  }
   if (option == OPRAG_OPT_PATH) {
     if (value < 0 || value > 2) return fail(OPRAG_ERR_INVALID_ARG, "path %d", value);
     if (value == 2 && idx->dtype != OPRAG_BF16)
