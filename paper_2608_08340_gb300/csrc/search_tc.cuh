@@ -861,9 +861,13 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
               constexpr int G = K / NC;         // groups per 32-column chunk
               static_assert(G >= 1 && 32 % G == 0, "group layout");
               float gmin = INFINITY;
-              auto group_min = [&](const uint32_t (&r)[32], int c) {
+#pragma unroll 1
+              for (int c = 0; c < NC; ++c) {
+                __syncwarp();
+                tmem_ld32_async(taddr + c * 32, ra);
+                tmem_wait_ld(ra);
                 float v[32];
-                scores(r, c, v);
+                scores(ra, c, v);
 #pragma unroll
                 for (int g = 0; g < G; ++g) {
                   constexpr int L = 32 / G;
@@ -873,17 +877,6 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                   if constexpr (L % 2 == 0) m = fmaxf(m, v[g * L + L - 1]);
                   gmin = fminf(gmin, m);
                 }
-              };
-              // Two chunks per TMEM round trip.
-#pragma unroll 1
-              for (int c = 0; c < NC; c += 2) {
-                __syncwarp();
-                tmem_ld32_async(taddr + c * 32, ra);
-                tmem_ld32_async(taddr + (c + 1) * 32, rb);
-                tmem_wait_ld(ra);
-                tmem_wait_ld(rb);
-                group_min(ra, c);
-                group_min(rb, c + 1);
               }
               bound = gmin;
             } else {
@@ -891,9 +884,13 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             constexpr int L = 32 / GPC;         // columns per group
             static_assert(GPC * NC == 32 && L >= 2, "group layout");
             float gm[32];
-            auto group_max = [&](const uint32_t (&r)[32], int c) {
+#pragma unroll
+            for (int c = 0; c < NC; ++c) {
+              __syncwarp();
+              tmem_ld32_async(taddr + c * 32, ra);
+              tmem_wait_ld(ra);
               float v[32];
-              scores(r, c, v);
+              scores(ra, c, v);
 #pragma unroll
               for (int g = 0; g < GPC; ++g) {
                 float m = v[g * L];
@@ -902,17 +899,6 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 if constexpr (L % 2 == 0) m = fmaxf(m, v[g * L + L - 1]);
                 gm[c * GPC + g] = m;
               }
-            };
-            // Two chunks per TMEM round trip.
-#pragma unroll
-            for (int c = 0; c < NC; c += 2) {
-              __syncwarp();
-              tmem_ld32_async(taddr + c * 32, ra);
-              tmem_ld32_async(taddr + (c + 1) * 32, rb);
-              tmem_wait_ld(ra);
-              tmem_wait_ld(rb);
-              group_max(ra, c);
-              group_max(rb, c + 1);
             }
             bitonic_desc32(gm);
             const int kk = p.k < 32 ? p.k : 32;
