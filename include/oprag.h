@@ -250,8 +250,12 @@ OPRAG_API int oprag_index_set_option(oprag_index *idx, int32_t option, int32_t v
 
 /* OPRAG_OPT_PAIR (tensor-core path): 2 runs clusters of two CTAs that issue
  * M = 256 MMAs together, each CTA loading half of every corpus tile (needs
- * 256-row corpus tiles; ignored with 128-row tiles).  0 (default) and 1 run
- * every CTA on its own (M = 128 MMAs). */
+ * 256-row corpus tiles; ignored with 128-row tiles).  1 runs every CTA on its
+ * own (M = 128 MMAs), one query tile per unit.  3 (dual mode) runs every CTA
+ * on its own with two query tiles per unit that share each corpus tile
+ * (256-row tiles; k <= 16 and more than 128 queries, ignored otherwise).
+ * 0 (default) chooses dual mode when its units fit in one wave of CTAs,
+ * single CTAs otherwise. */
 #define OPRAG_OPT_PAIR 4
 
 /* OPRAG_OPT_BOUND_TAG (test hook): sets the 32-bit tag of the last search's
@@ -294,6 +298,11 @@ OPRAG_API int oprag_index_last_path(const oprag_index *idx);
  * Out-pointers may be NULL.  OPRAG_ERR_NOT_READY before the first search. */
 OPRAG_API int oprag_index_last_launch(const oprag_index *idx, int32_t *grid, int32_t *cluster,
                                       int32_t *block_n);
+
+/* Query tiles (of 128 queries) that one CTA of the last search's main
+ * tensor-core kernel takes per unit: 2 in dual mode (OPRAG_OPT_PAIR), else 1;
+ * 0 for the SIMT kernel.  OPRAG_ERR_NOT_READY before the first search. */
+OPRAG_API int oprag_index_last_tiles_per_cta(const oprag_index *idx, int32_t *tiles);
 
 /*
  * oprag_search without any device allocation.  The paper has no counterpart:

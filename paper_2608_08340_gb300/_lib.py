@@ -58,6 +58,7 @@ SIGNATURES = {
     "oprag_index_last_path": (_I32, [_P]),
     "oprag_index_last_launch": (_I32, [_P, ctypes.POINTER(_I32), ctypes.POINTER(_I32),
                                        ctypes.POINTER(_I32)]),
+    "oprag_index_last_tiles_per_cta": (_I32, [_P, ctypes.POINTER(_I32)]),
     "oprag_index_last_timing": (_I32, [_P, ctypes.POINTER(_F), ctypes.POINTER(_F),
                                        ctypes.POINTER(_F)]),
     "oprag_last_error": (ctypes.c_char_p, []),

@@ -64,6 +64,7 @@ struct TcPlan {
   int block_n;     // corpus rows per tile: 128 or 256
   int grid;        // CTAs (persistent)
   int pair;        // 2: clusters of two CTAs issue M = 256 MMAs together; 1: single CTAs
+  bool dual;       // single CTAs that take two query tiles per unit (see search_tc.cuh)
   int qt;          // query tiles of 128
   int uqt;         // query tiles of the schedule: qt, or ceil(qt / 2) pairs of tiles
   int nt;          // corpus tiles
@@ -74,7 +75,8 @@ struct TcPlan {
   size_t smem;
 };
 // tile_stride > 1 scans only corpus tiles t = 0, stride, 2 * stride, ...
-// force_pair: 0 automatic, 1 single CTAs, 2 CTA pairs (needs 256-row tiles).
+// force_pair: 0 automatic, 1 single CTAs, 2 CTA pairs (needs 256-row tiles),
+// 3 dual mode (single CTAs, two query tiles per unit; lists of 8 or 16).
 // pair_capacity: clusters of two that fit on the device (0: no pair mode).
 TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_stride = 1,
                int force_pair = 0, int pair_capacity = 0);

@@ -5,8 +5,9 @@
 // are corpus slices instead of index shards.
 //
 // Three merges by list count and k: one warp per query over at most 32
-// sorted lists (head by head), one warp per query over more lists when
-// k <= 16, and the block merge of merge.cuh (one CTA per query) otherwise.
+// sorted lists (head by head), one to four warps per query over up to 384
+// lists when k <= 16 (also head by head), and the block merge of merge.cuh
+// (one CTA per query) otherwise.
 #include "merge.cuh"
 
 namespace oprag {
@@ -113,67 +114,89 @@ merge_kway_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
   }
 }
 
-// More than 32 lists and k <= 16: one warp per query, two queries per CTA of
-// 64 threads with at most 64 registers a thread, so that a CTA fits on an SM
-// beside a running search CTA: launched early (programmatic dependent launch),
-// it waits in place and starts as soon as the search grid ends.  Lane l reads
-// the keys l, l + 32, ... of the query's np * kl candidates (64 / KL
-// independent loads at a time, within the register budget) and keeps the
-// best KL sorted in registers;
-// then the lanes' sorted lists are merged head by head as above.
-constexpr int kSmallWarps = 2;
+// More than 32 lists and k <= 16, at most kSmallLists lists per lane: W
+// warps per query (W = 4, 2 or 1; CTAs of four warps, 4 / W queries each).
+// Launched early (programmatic dependent
+// launch), a CTA waits in place and starts as soon as the search grid ends.
+// Lane l of warp w holds lists p = 32 w + l + 32 W u (u < kSmallLists): the
+// first kSmallKeys keys of each, fetched with 16-byte loads all issued
+// together.  Then the query's 32 W lanes take the k best head by head:
+// each round the lanes' best heads go through a warp maximum (and, when
+// W > 1, a maximum over the query's warps in shared memory); keys are
+// unique, so one lane owns the winner and advances that list (fetching its
+// next keys once the held ones are used up, which only k > kSmallKeys can
+// need).
+constexpr int kSmallThreads = 128;
+constexpr int kSmallLists = 3;
+constexpr int kSmallKeys = 6;
 
-template <int KL>
-__global__ void __launch_bounds__(kSmallWarps * 32, 16)
+template <int W>
+__global__ void __launch_bounds__(kSmallThreads, 4)
 merge_small_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
                    float* __restrict__ out_scores, float* __restrict__ kth_out,
                    float* __restrict__ levels_out) {
+  constexpr int kQPerCta = kSmallThreads / 32 / W;
+  __shared__ uint64_t heads[2][kSmallThreads / 32];
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int qi = blockIdx.x * kSmallWarps + warp;
-  if (qi >= q) return;
+  const int qs = warp / W, wq = warp % W;      // query slot in the CTA, warp of the query
+  const int qi = blockIdx.x * kQPerCta + qs;
+  if (qi >= q) return;                         // all W warps of the slot leave together
   const int tile = qi / ls.TH, row = qi % ls.TH;
   const int np = merge_list_count(ls, tile);
   const int kl = min(k, ls.klen);
-  const int total = np * kl;
   const uint64_t* base = ls.keys + (static_cast<int64_t>(tile) * ls.P * ls.TH + row) * ls.stride;
   const int64_t list_step = static_cast<int64_t>(ls.TH) * ls.stride;
-  constexpr int kLoadBatch = 64 / KL;
-  uint64_t top[KL];
+  // Keys at or past kl of a list are not candidates; a missing list is empty.
+  auto fetch = [&](int u, int from, uint64_t (&dst)[kSmallKeys]) {
+    const int p = wq * 32 + lane + u * 32 * W;
+    const uint64_t* l = base + p * list_step + from;
 #pragma unroll
-  for (int i = 0; i < KL; ++i) top[i] = kEmptyKey;
-  for (int g = lane; g < total; g += 32 * kLoadBatch) {
-    uint64_t key[kLoadBatch];
-#pragma unroll
-    for (int u = 0; u < kLoadBatch; ++u) {
-      const int i = g + 32 * u;
-      key[u] = kEmptyKey;
-      if (i < total) {
-        const int pl = i / kl;
-        key[u] = base[pl * list_step + (i - pl * kl)];
-      }
+    for (int j = 0; j < kSmallKeys; j += 2) {
+      ulonglong2 v = make_ulonglong2(kEmptyKey, kEmptyKey);
+      if (p < np && from + j < kl) v = *reinterpret_cast<const ulonglong2*>(l + j);
+      dst[j] = v.x;
+      dst[j + 1] = from + j + 1 < kl ? v.y : kEmptyKey;
     }
+  };
+  uint64_t key[kSmallLists][kSmallKeys];
+  int used[kSmallLists];
 #pragma unroll
-    for (int u = 0; u < kLoadBatch; ++u) {
-      const uint64_t x = key[u];
-      if (x > top[KL - 1]) {
-#pragma unroll
-        for (int i = KL - 1; i > 0; --i)
-          top[i] = x > top[i - 1] ? top[i - 1] : (x > top[i] ? x : top[i]);
-        top[0] = x > top[0] ? x : top[0];
-      }
-    }
+  for (int u = 0; u < kSmallLists; ++u) {
+    fetch(u, 0, key[u]);
+    used[u] = 0;
   }
   uint64_t mine = kEmptyKey;
   for (int r = 0; r < k; ++r) {
-    uint64_t best = top[0];
+    uint64_t own = key[0][0];
+#pragma unroll
+    for (int u = 1; u < kSmallLists; ++u) own = umax64(own, key[u][0]);
+    uint64_t best = own;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) best = umax64(best, __shfl_xor_sync(0xffffffffu, best, o));
-    if (best != kEmptyKey && top[0] == best) {
+    if constexpr (W > 1) {
+      if (lane == 0) heads[r & 1][warp] = best;
+      // The query's W warps (named barrier 1 + slot; constant ids, so
+      // that the kernel reserves only the barriers it uses).
+      if (qs == 0) asm volatile("bar.sync 1, %0;" ::"n"(32 * W) : "memory");
+      else asm volatile("bar.sync 2, %0;" ::"n"(32 * W) : "memory");
 #pragma unroll
-      for (int i = 0; i + 1 < KL; ++i) top[i] = top[i + 1];
-      top[KL - 1] = kEmptyKey;
+      for (int j = 0; j < W; ++j) best = umax64(best, heads[r & 1][qs * W + j]);
     }
+    if (best != kEmptyKey && own == best) {
+      bool done = false;
+#pragma unroll
+      for (int u = 0; u < kSmallLists; ++u) {
+        if (!done && key[u][0] == best) {
+          done = true;
+#pragma unroll
+          for (int j = 0; j + 1 < kSmallKeys; ++j) key[u][j] = key[u][j + 1];
+          key[u][kSmallKeys - 1] = kEmptyKey;
+          if (++used[u] % kSmallKeys == 0 && used[u] < kl) fetch(u, used[u], key[u]);
+        }
+      }
+    }
+    if (wq != 0) continue;
     if ((r & 31) == lane) mine = best;
     if ((r & 31) == 31 || r == k - 1) {
       const int i = (r & ~31) + lane;
@@ -206,6 +229,41 @@ cudaError_t launch_warp_per_query(Kern kern, int warps, const ListSet& ls, int q
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kern, ls, q, k, out_ids, out_scores, kth_out, levels_out);
+}
+
+template <int W>
+cudaError_t launch_small_w(const ListSet& ls, int q, int k, int64_t* out_ids, float* out_scores,
+                           cudaStream_t st, float* kth_out, float* levels_out) {
+  constexpr int kQPerCta = kSmallThreads / 32 / W;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((q + kQPerCta - 1) / kQPerCta);
+  cfg.blockDim = dim3(kSmallThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, merge_small_kernel<W>, ls, q, k, out_ids, out_scores, kth_out,
+                            levels_out);
+}
+
+// Warps per query of merge_small_kernel: four while one merge CTA per SM
+// covers the batch, else two, else one.  Returns cudaErrorNotSupported when
+// a lane would hold more than kSmallLists lists (the caller then takes the
+// block merge).
+cudaError_t launch_small(const ListSet& ls, int q, int k, int64_t* out_ids, float* out_scores,
+                         cudaStream_t st, float* kth_out, float* levels_out) {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    sms = 1;
+  const int W = q <= sms ? 4 : q <= 2 * sms ? 2 : 1;
+  if (ls.P > kSmallLists * 32 * W) return cudaErrorNotSupported;
+  if (W == 4) return launch_small_w<4>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
+  if (W == 2) return launch_small_w<2>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
+  return launch_small_w<1>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
 }
 
 }  // namespace
@@ -268,12 +326,10 @@ cudaError_t launch_merge(const ListSet& ls, int q, int k, int64_t* out_ids, floa
   if (ls.P <= 32)
     return launch_warp_per_query(merge_kway_kernel, kWayWarps, ls, q, k, out_ids, out_scores, st,
                                  kth_out, levels_out);
-  if (k <= 8)
-    return launch_warp_per_query(merge_small_kernel<8>, kSmallWarps, ls, q, k, out_ids,
-                                 out_scores, st, kth_out, levels_out);
-  if (k <= 16)
-    return launch_warp_per_query(merge_small_kernel<16>, kSmallWarps, ls, q, k, out_ids,
-                                 out_scores, st, kth_out, levels_out);
+  if (k <= 16) {
+    const cudaError_t e = launch_small(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
+    if (e != cudaErrorNotSupported) return e;
+  }
   if (k <= 32) return launch_merge_kp<32>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
   if (k <= 64) return launch_merge_kp<64>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
   if (k <= 128) return launch_merge_kp<128>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);

@@ -121,6 +121,7 @@ struct oprag_index {
   int pair_cap = -1;       // clusters of two search CTAs that fit at once (-1: not asked yet)
   int last_path = 0;
   int last_grid = 0, last_cluster = 0, last_block_n = 0;   // last main search kernel launch
+  int last_tiles = 0;                                         // query tiles per CTA and unit
 
   // Optional kernel timing: events before the lexical pass, before the
   // search kernel, before the merge kernel and after it.
@@ -225,8 +226,9 @@ void note_launch(oprag_index* idx, int path, const TcPlan& plan) {
     idx->last_grid = plan.grid;
     idx->last_cluster = plan.pair;
     idx->last_block_n = plan.block_n;
+    idx->last_tiles = plan.dual ? 2 : 1;
   } else {
-    idx->last_grid = idx->last_cluster = idx->last_block_n = 0;
+    idx->last_grid = idx->last_cluster = idx->last_block_n = idx->last_tiles = 0;
   }
 }
 
@@ -474,7 +476,7 @@ int oprag_index_reserve(oprag_index* idx, int32_t q_max, int32_t k_max) {
       for (int qq : {q_max, std::min(q_max, 128)}) {
         SearchShape s2 = s;
         s2.q = qq;
-        for (int pair : {1, 2})
+        for (int pair : {1, 2, 3})
           need = std::max(need, tc_scratch_bytes(s2, tc_plan(s2, idx->num_sms, bn, 1, pair,
                                                              pair_capacity(idx))));
       }
@@ -1040,7 +1042,7 @@ int oprag_index_set_option(oprag_index* idx, int32_t option, int32_t value) {
     return ok();
   }
   if (option == OPRAG_OPT_PAIR) {
-    if (value < 0 || value > 2) return fail(OPRAG_ERR_INVALID_ARG, "pair mode %d", value);
+    if (value < 0 || value > 3) return fail(OPRAG_ERR_INVALID_ARG, "pair mode %d", value);
     idx->opt_pair = value;
     return ok();
   }
@@ -1062,6 +1064,13 @@ int oprag_index_last_launch(const oprag_index* idx, int32_t* grid, int32_t* clus
   if (grid) *grid = idx->last_grid;
   if (cluster) *cluster = idx->last_cluster;
   if (block_n) *block_n = idx->last_block_n;
+  return ok();
+}
+
+int oprag_index_last_tiles_per_cta(const oprag_index* idx, int32_t* tiles) {
+  if (!idx) return fail(OPRAG_ERR_INVALID_ARG, "index is NULL");
+  if (!idx->last_path) return fail(OPRAG_ERR_NOT_READY, "no search was issued");
+  if (tiles) *tiles = idx->last_tiles;
   return ok();
 }
 

@@ -64,6 +64,17 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
     const int64_t units256 = static_cast<int64_t>(pl.qt) * ((s.n + 255) / 256);
     if (units256 < 4LL * num_sms) bn = 128;
   }
+  // Dual mode: every unit takes two query tiles and one 256-row corpus tile,
+  // so a CTA reads each corpus tile once for 256 queries.  Automatic when
+  // there are at least two query tiles and the dual units fit in one wave
+  // (small batches, where the copies into the SMs, not the MMAs, bound the
+  // kernel and no unit's epilogue has a next unit to overlap); it needs the
+  // two epilogue sets of lists of 8 or 16.
+  const bool dual_ok = pl.qt >= 2 && epi_sets(list_len_for(s.k)) == 2 && force_pair != 2 &&
+                       (force_block_n == 0 || force_block_n == 256);
+  const int64_t dual_units = static_cast<int64_t>((pl.qt + 1) / 2) * ((s.n + 255) / 256);
+  pl.dual = dual_ok && (force_pair == 3 || (force_pair == 0 && dual_units <= num_sms));
+  if (pl.dual) bn = 256;
   pl.block_n = bn;
   // CTA pairs cut the operand bytes each SM loads per MMA by a third; they
   // need 256-row corpus tiles and a device that fits clusters of two.  They
@@ -72,7 +83,7 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
   // not operand bytes, bound the kernel).
   const bool pair = bn == 256 && pair_capacity > 0 && force_pair == 2;
   pl.pair = pair ? 2 : 1;
-  pl.uqt = pair ? (pl.qt + 1) / 2 : pl.qt;
+  pl.uqt = pair || pl.dual ? (pl.qt + 1) / 2 : pl.qt;
   pl.tile_stride = tile_stride < 1 ? 1 : tile_stride;
   const int64_t all_tiles = (s.n + bn - 1) / bn;
   pl.nt = static_cast<int>((all_tiles + pl.tile_stride - 1) / pl.tile_stride);
@@ -112,20 +123,23 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
   for (int j = 0; j < pl.uqt; ++j)
     per_tile = std::max(per_tile, hi[j] - first_cta(j, pl.uqt, C) + 1);
   if (!ok) per_tile = C;  // not expected; every slot then gets a list per tile
-  pl.pmax = per_tile * epi_sets(list_len_for(s.k));
+  pl.pmax = per_tile * (pl.dual ? 1 : epi_sets(list_len_for(s.k)));
   const int K = list_len_for(s.k);
-  // Shared memory of the launch (the same sum as smem_for<BN, K, pair>).
+  // Shared memory of the launch (the same sum as smem_for<BN, K, pair, dual>).
   const size_t b_stage = static_cast<size_t>(pair ? bn / 2 : bn) * 128;
-  pl.stages = pair ? stages_for<256, true>() : (bn == 128 ? stages_for<128>() : stages_for<256>());
-  pl.smem = static_cast<size_t>(pl.stages) * (kAStageBytes + b_stage) +
+  const size_t a_stage = kAStageBytes * (pl.dual ? 2 : 1);
+  pl.stages = pair      ? stages_for<256, true>()
+              : pl.dual ? stages_for<256, false, true>()
+                        : (bn == 128 ? stages_for<128>() : stages_for<256>());
+  pl.smem = static_cast<size_t>(pl.stages) * (a_stage + b_stage) +
             static_cast<size_t>(epi_sets(K)) * 128 * kStageRowBytes + 1024 + 256;
   return pl;
 }
 
-// List rows: one per (query tile, producer, query row); pair mode covers
-// 2 * uqt tiles (an odd qt leaves the last pair's second tile empty).
+// List rows: one per (query tile, producer, query row); pair and dual modes
+// cover 2 * uqt tiles (an odd qt leaves the last pair's second tile empty).
 static size_t list_rows(const TcPlan& pl) {
-  return static_cast<size_t>(pl.uqt) * pl.pair * pl.pmax * kBlockM;
+  return static_cast<size_t>(pl.uqt) * (pl.pair == 2 || pl.dual ? 2 : 1) * pl.pmax * kBlockM;
 }
 
 size_t tc_scratch_bytes(const SearchShape& s, const TcPlan& pl) {
@@ -147,7 +161,8 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
   // reads); rows are loaded in multiples of 8, the swizzle atom height.
   // Pair mode: each CTA loads all 128 rows of its tile and half of the
   // corpus tile.
-  const int a_rows = pl.qt == 1 && pl.pair == 1 ? std::min(kBlockM, (s.q + 7) / 8 * 8) : kBlockM;
+  const int a_rows =
+      pl.qt == 1 && pl.pair == 1 && !pl.dual ? std::min(kBlockM, (s.q + 7) / 8 * 8) : kBlockM;
   if (!make_map(&mq, Q, s.q, s.d, a_rows) ||
       !make_map(&me, E, s.n, s.d, pl.block_n / pl.pair))
     return cudaErrorInvalidValue;
@@ -183,10 +198,14 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
   lists->stride = stride;
   lists->C = pl.grid / pl.pair;
   lists->qt = pl.uqt;
-  lists->sets = epi_sets(K);
+  lists->sets = pl.dual ? 1 : epi_sets(K);
   lists->klen = K;
-  lists->pair = pl.pair;
+  lists->pair = pl.dual ? 2 : pl.pair;
   const bool hybrid = fu.bm25 != nullptr;
+  if (pl.dual) {
+    if (pl.block_n != 256) return cudaErrorInvalidValue;
+    return launch_dual256(mq, me, prm, pl.grid, hybrid, st);
+  }
   if (pl.pair == 2) {
     if (pl.block_n != 256) return cudaErrorInvalidValue;
     return hybrid ? launch_pair256_fused(mq, me, prm, pl.grid, st)

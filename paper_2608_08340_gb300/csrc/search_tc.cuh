@@ -138,20 +138,27 @@ constexpr uint32_t b_stage_bytes() {
   return static_cast<uint32_t>(kPair ? BN / 2 : BN) * 128;
 }
 
-template <int BN, bool kPair = false>
+// Query rows per stage: one 128-row tile, or two in dual mode.
+template <bool kDual>
+constexpr uint32_t a_stage_bytes() {
+  return kAStageBytes * (kDual ? 2u : 1u);
+}
+
+template <int BN, bool kPair = false, bool kDual = false>
 constexpr int stages_for() {
-  return kSmemBudget / (kAStageBytes + b_stage_bytes<BN, kPair>()) > 8
+  return kSmemBudget / (a_stage_bytes<kDual>() + b_stage_bytes<BN, kPair>()) > 8
              ? 8
-             : kSmemBudget / (kAStageBytes + b_stage_bytes<BN, kPair>());
+             : kSmemBudget / (a_stage_bytes<kDual>() + b_stage_bytes<BN, kPair>());
 }
 
 // Per epilogue thread: one 32-float row where a chunk's scores are staged so
 // that candidate columns can be read back by index.
 constexpr int kStageRowBytes = 32 * 4;
 
-template <int BN, int K, bool kPair = false>
+template <int BN, int K, bool kPair = false, bool kDual = false>
 constexpr size_t smem_for() {
-  return static_cast<size_t>(stages_for<BN, kPair>()) * (kAStageBytes + b_stage_bytes<BN, kPair>()) +
+  return static_cast<size_t>(stages_for<BN, kPair, kDual>()) *
+             (a_stage_bytes<kDual>() + b_stage_bytes<BN, kPair>()) +
          static_cast<size_t>(epi_sets(K)) * 128 * kStageRowBytes + 1024 + 256;
 }
 
@@ -369,12 +376,13 @@ __device__ __forceinline__ void shared_floor_raise(uint64_t* qf, int64_t qi, uin
             (static_cast<unsigned long long>(gen) << 32) | ordered_bits(f));
 }
 
-// Sorts 32 values descending in registers (bitonic network, 240 exchanges);
-// the stages are template instances so that every index is a constant.
-template <int KS, int JS>
-__device__ __forceinline__ void bitonic_stage32(float (&a)[32]) {
+// Sorts N (a power of two) values descending in registers (bitonic network;
+// 240 exchanges for N = 32); the stages are template instances so that every
+// index is a constant.
+template <int N, int KS, int JS>
+__device__ __forceinline__ void bitonic_stage(float (&a)[N]) {
 #pragma unroll
-  for (int i = 0; i < 32; ++i) {
+  for (int i = 0; i < N; ++i) {
     const int l = i ^ JS;
     if (l > i) {
       const float hi = fmaxf(a[i], a[l]), lo = fminf(a[i], a[l]);
@@ -383,13 +391,14 @@ __device__ __forceinline__ void bitonic_stage32(float (&a)[32]) {
       a[l] = desc ? lo : hi;
     }
   }
-  if constexpr (JS > 1) bitonic_stage32<KS, JS / 2>(a);
+  if constexpr (JS > 1) bitonic_stage<N, KS, JS / 2>(a);
 }
 
-template <int KS = 2>
-__device__ __forceinline__ void bitonic_desc32(float (&a)[32]) {
-  bitonic_stage32<KS, KS / 2>(a);
-  if constexpr (KS < 32) bitonic_desc32<KS * 2>(a);
+template <int N, int KS = 2>
+__device__ __forceinline__ void bitonic_desc(float (&a)[N]) {
+  static_assert(N >= 2 && (N & (N - 1)) == 0, "power of two");
+  bitonic_stage<N, KS, KS / 2>(a);
+  if constexpr (KS < N) bitonic_desc<N, KS * 2>(a);
 }
 
 // Three-input maximum (one instruction on sm_100 and later).
@@ -433,20 +442,63 @@ struct EpiList;
 template <int K>
 struct EpiList<K, false> {
   static constexpr int kStride = K;
+  // Only the best kk = min(k, K) keys of a list can reach the query's top-k
+  // (the merges read no more).  The list keeps them in its last kk slots,
+  // under pad = K - kk sentinel slots of +inf that no score passes, so the
+  // insertion network is unchanged and the floor (the last slot) is the
+  // kk-th best score.  Stored lists hold their kk keys first.
   RegTopK<K> t;
+  int pad = 0;
+  __device__ __forceinline__ void set_k(int k) { pad = k < K ? K - k : 0; }
   __device__ __forceinline__ void init_mem(const TcParams& p, int64_t sr, int) {
 #pragma unroll
     for (int i = 0; i < K; i += 2)
       *reinterpret_cast<ulonglong2*>(p.lists + sr * K + i) = make_ulonglong2(0ull, 0ull);
   }
-  __device__ __forceinline__ void load(const TcParams& p, int64_t sr) { t.load(p.lists + sr * K); }
-  __device__ __forceinline__ void save(const TcParams& p, int64_t sr) { t.store(p.lists + sr * K); }
-  __device__ __forceinline__ void clear() { t.init(); }
+  __device__ __forceinline__ void pad_top() {
+#pragma unroll
+    for (int i = 0; i + 1 < K; ++i)
+      if (i < pad) t.s[i] = INFINITY;
+  }
+  // Stored order -> slots: shift right by pad (a barrel shifter, so that
+  // every register index is a constant).
+  __device__ __forceinline__ void load(const TcParams& p, int64_t sr) {
+    t.load(p.lists + sr * K);
+#pragma unroll
+    for (int w = K / 2; w >= 1; w /= 2) {
+      const bool on = (pad & w) != 0;
+#pragma unroll
+      for (int j = K - 1; j >= 0; --j) {
+        t.s[j] = on ? (j >= w ? t.s[j - w] : INFINITY) : t.s[j];
+        t.id[j] = on ? (j >= w ? t.id[j - w] : kNoId) : t.id[j];
+      }
+    }
+    t.floor = t.s[K - 1];
+  }
+  // Slots -> stored order: shift left by pad, empty keys behind.
+  __device__ __forceinline__ void save(const TcParams& p, int64_t sr) {
+    RegTopK<K> o = t;
+#pragma unroll
+    for (int w = 1; w <= K / 2; w *= 2) {
+      const bool on = (pad & w) != 0;
+#pragma unroll
+      for (int j = 0; j < K; ++j) {
+        o.s[j] = on ? (j + w < K ? o.s[j + w] : -INFINITY) : o.s[j];
+        o.id[j] = on ? (j + w < K ? o.id[j + w] : kNoId) : o.id[j];
+      }
+    }
+    o.store(p.lists + sr * K);
+  }
+  __device__ __forceinline__ void clear() {
+    t.init();
+    pad_top();
+  }
   __device__ __forceinline__ bool full() const { return t.full(); }
   __device__ __forceinline__ float floor() const { return t.floor; }
   __device__ __forceinline__ void push(float s, uint32_t id) { t.push(s, id); }
   __device__ __forceinline__ void insert(float s, uint32_t id) { t.insert(s, id); }
-  __device__ __forceinline__ float kth(int k) const { return t.kth(k); }
+  // The k-th best score held, for the k the list was set up with.
+  __device__ __forceinline__ float kth(int) const { return t.floor; }
   __device__ __forceinline__ void sync(bool, bool) {}
   __device__ __forceinline__ void finalize(const TcParams&, int64_t, bool) {}
 };
@@ -490,6 +542,7 @@ struct EpiList<K, true> {
     p.meta_count[sr] = t.count;
     p.meta_worst[sr] = t.worst;
   }
+  __device__ __forceinline__ void set_k(int) {}
   __device__ __forceinline__ void clear() {
     t.buf = nullptr;
     t.count = 0;
@@ -532,11 +585,21 @@ struct EpiList<K, true> {
 // MMA each CTA then reads 128 x 16 + BN / 2 x 16 operand elements instead of
 // 128 x 16 + BN x 16.  The unit sequence (UnitSeq) runs over pairs: p.qt
 // counts pairs of query tiles and the pair index plays the CTA index.
-template <int BN, int K, bool kHybrid, bool kPair = false>
+//
+// kDual: every unit covers query tiles 2J and 2J + 1 and corpus tile t; a
+// stage holds both query tiles' K-block and the corpus tile's, and the MMA
+// warp issues two MMAs per K-step that share the corpus operand, one into
+// each accumulator.  Epilogue set s filters query tile 2J + s.  Per unit the
+// CTA reads the corpus tile once for 256 queries, so small batches (one unit
+// per CTA) load half the operand bytes of two single-tile units.
+template <int BN, int K, bool kHybrid, bool kPair = false, bool kDual = false>
 __global__ void __launch_bounds__(threads_for(K), 1)
 tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_e,
                  const TcParams p) {
-  constexpr int S = stages_for<BN, kPair>();
+  static_assert(!(kPair && kDual), "pair and dual modes are exclusive");
+  static_assert(!kDual || epi_sets(K) == 2, "dual mode needs one epilogue set per query tile");
+  constexpr int S = stages_for<BN, kPair, kDual>();
+  constexpr uint32_t kAStage = a_stage_bytes<kDual>();
   constexpr uint32_t kBStageBytes = b_stage_bytes<BN, kPair>();
   constexpr uint32_t kTmemCols = 2 * BN;
   constexpr int kEpiSets = epi_sets(K);
@@ -544,7 +607,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
   unsigned char* base = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   unsigned char* sA = base;
-  unsigned char* sB = sA + S * kAStageBytes;
+  unsigned char* sB = sA + S * kAStage;
   float* stage_rows = reinterpret_cast<float*>(sB + S * kBStageBytes);   // epilogue staging
   uint64_t* full = reinterpret_cast<uint64_t*>(stage_rows + kEpiSets * 128 * 32);
   uint64_t* empty = full + S;
@@ -562,9 +625,11 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
   const int cta = kPair ? static_cast<int>(cluster_index()) : static_cast<int>(blockIdx.x);
   const int C = kPair ? static_cast<int>(gridDim.x) / 2 : static_cast<int>(gridDim.x);
   // Bytes one stage brings into the leader's full barrier (both CTAs in pair mode).
-  const uint32_t stage_tx = (p.a_bytes + kBStageBytes) * (kPair ? 2u : 1u);
+  const uint32_t stage_tx = (p.a_bytes * (kDual ? 2u : 1u) + kBStageBytes) * (kPair ? 2u : 1u);
   // Row coordinates of this CTA's part of unit (J, t).
-  auto a_row = [&](int J) { return (kPair ? 2 * J + static_cast<int>(rank) : J) * kBlockM; };
+  auto a_row = [&](int J) {
+    return (kPair ? 2 * J + static_cast<int>(rank) : kDual ? 2 * J : J) * kBlockM;
+  };
   auto b_row = [&](int t) {
     return t * BN + (kPair ? static_cast<int>(rank) * (BN / 2) : 0);
   };
@@ -591,11 +656,14 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     if (kPair) {
       if (leader) mbar_arrive_expect_tx(&full[s], stage_tx);
       const uint32_t bar = cluster_addr(&full[s], 0);                  // the leader's full[s]
-      tma_load_2d_pair(sA + s * kAStageBytes, &map_q, bar, kb * kBlockK, a_row(J));
+      tma_load_2d_pair(sA + s * kAStage, &map_q, bar, kb * kBlockK, a_row(J));
       tma_load_2d_pair(sB + s * kBStageBytes, &map_e, bar, kb * kBlockK, b_row(t));
     } else {
       mbar_arrive_expect_tx(&full[s], stage_tx);
-      tma_load_2d(sA + s * kAStageBytes, &map_q, &full[s], kb * kBlockK, a_row(J));
+      tma_load_2d(sA + s * kAStage, &map_q, &full[s], kb * kBlockK, a_row(J));
+      if constexpr (kDual)
+        tma_load_2d(sA + s * kAStage + kAStageBytes, &map_q, &full[s], kb * kBlockK,
+                    a_row(J) + kBlockM);
       tma_load_2d(sB + s * kBStageBytes, &map_e, &full[s], kb * kBlockK, b_row(t));
     }
   };
@@ -666,13 +734,39 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       bool ok = true;
       UnitSeq us;
       for (us.start(p, cta, C); ok && us.valid(); us.next()) {
+        if constexpr (kDual) {
+          // Both accumulators take this unit.
+          if (!mbar_wait(&tempty[0], acc_ph ^ 1u, abort_flag, p.dev_err)) break;
+          if (!mbar_wait(&tempty[1], acc_ph ^ 1u, abort_flag, p.dev_err)) break;
+          tc_fence_after();
+          for (int kb = 0; kb < p.kblocks; ++kb) {
+            if (!mbar_wait(&full[s], ph, abort_flag, p.dev_err)) { ok = false; break; }
+            tc_fence_after();
+            const uint64_t a0 = sw128_desc(smem_addr(sA + s * kAStage));
+            const uint64_t a1 = sw128_desc(smem_addr(sA + s * kAStage + kAStageBytes));
+            const uint64_t b = sw128_desc(smem_addr(sB + s * kBStageBytes));
+#pragma unroll
+            for (int kk = 0; kk < kBlockK / kUmmaK; ++kk) {
+              const uint32_t accum = (kb | kk) != 0 ? 1u : 0u;
+              mma_bf16(tmem_base, a0 + 2 * kk, b + 2 * kk, idesc, accum);
+              mma_bf16(tmem_base + static_cast<uint32_t>(BN), a1 + 2 * kk, b + 2 * kk, idesc, accum);
+            }
+            mma_commit(&empty[s]);
+            if (++s == S) { s = 0; ph ^= 1u; }
+          }
+          if (!ok) break;
+          mma_commit(&tfull[0]);
+          mma_commit(&tfull[1]);
+          acc_ph ^= 1u;
+          continue;
+        }
         if (!mbar_wait<kPair>(&tempty[acc], acc_ph ^ 1u, abort_flag, p.dev_err)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
         for (int kb = 0; kb < p.kblocks; ++kb) {
           if (!mbar_wait(&full[s], ph, abort_flag, p.dev_err)) { ok = false; break; }
           tc_fence_after();
-          const uint64_t a = sw128_desc(smem_addr(sA + s * kAStageBytes));
+          const uint64_t a = sw128_desc(smem_addr(sA + s * kAStage));
           const uint64_t b = sw128_desc(smem_addr(sB + s * kBStageBytes));
           if constexpr (kPair) {
 #pragma unroll
@@ -701,22 +795,28 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     // ------------------------------------------------ epilogue
     // kEpiSets sets of four warps; set s filters the units whose sequence
     // number is s modulo kEpiSets (with two sets, two units are filtered at
-    // the same time).  Each set keeps its own lists.
+    // the same time).  Each set keeps its own lists.  Dual mode: set s
+    // filters query tile 2J + s of every unit, from accumulator s.
     const int set = (warp - 2) >> 2;
     const int eg = warp & 3;                 // TMEM lane group of this warp
     const int row = eg * 32 + lane;          // query row within a tile
-    const int per_tile = p.pmax / kEpiSets;  // CTAs (pairs) per unit query tile with a list slot
+    constexpr int kRowSets = kDual ? 1 : kEpiSets;   // list slots per producer and tile
+    const int per_tile = p.pmax / kRowSets;  // CTAs (pairs) per unit query tile with a list slot
     // Unit query tile J covers this CTA's query tile qtile(J) (one of a pair's two).
-    auto qtile = [&](int J) { return kPair ? 2 * J + static_cast<int>(rank) : J; };
+    auto qtile = [&](int J) {
+      return kPair ? 2 * J + static_cast<int>(rank) : kDual ? 2 * J + set : J;
+    };
     auto list_row = [&](int J) -> int64_t {
       const int pc = cta - first_cta(J, p.qt, C);
-      return (static_cast<int64_t>(qtile(J)) * p.pmax + pc * kEpiSets + set) * kBlockM + row;
+      return (static_cast<int64_t>(qtile(J)) * p.pmax + pc * kRowSets + (kDual ? 0 : set)) *
+                 kBlockM + row;
     };
     auto owns = [&](int J) {
       const int pc = cta - first_cta(J, p.qt, C);
       return pc >= 0 && pc < per_tile;
     };
     EpiList<K> list;
+    list.set_k(p.k);
     list.clear();
 
     // This CTA owns the list slots (J, cta - first_cta(J)); empty them first.
@@ -732,8 +832,8 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     UnitSeq us;
     int seq = 0;
     for (us.start(p, cta, C); us.valid(); us.next(), ++seq) {
-      if (seq % kEpiSets != set) continue;
-      const int acc = seq & 1;
+      if (!kDual && seq % kEpiSets != set) continue;
+      const int acc = kDual ? set : (seq & 1);
       const int J = us.j();
       const int j = qtile(J);                // this CTA's query tile
       const int64_t t = us.t();
@@ -856,11 +956,13 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             // score below it can be among the query's k best.  Lists of 16
             // or 32 use 32 groups and sort their maxima (a tight bound pays
             // for the sort when each insertion costs 16-32 steps); lists of
-            // 8 use K groups and the smallest maximum, which needs no sort.
+            // 8 use 8 groups (a sort of 8 values).
             if constexpr (K <= 8) {
               constexpr int G = K / NC;         // groups per 32-column chunk
               static_assert(G >= 1 && 32 % G == 0, "group layout");
-              float gmin = INFINITY;
+              // Group maxima enter gm through a shift (constant indices in a
+              // loop that is not unrolled).
+              float gm[K];
 #pragma unroll 1
               for (int c = 0; c < NC; ++c) {
                 __syncwarp();
@@ -869,16 +971,20 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 float v[32];
                 scores(ra, c, v);
 #pragma unroll
+                for (int i = K - 1; i >= G; --i) gm[i] = gm[i - G];
+#pragma unroll
                 for (int g = 0; g < G; ++g) {
                   constexpr int L = 32 / G;
                   float m = v[g * L];
 #pragma unroll
                   for (int i = 1; i + 1 < L; i += 2) m = fmax3(m, v[g * L + i], v[g * L + i + 1]);
                   if constexpr (L % 2 == 0) m = fmaxf(m, v[g * L + L - 1]);
-                  gmin = fminf(gmin, m);
+                  gm[g] = m;
                 }
               }
-              bound = gmin;
+              // The k-th largest group maximum (K groups, k <= K).
+              bitonic_desc<K>(gm);
+              bound = reg_select(gm, (p.k < K ? p.k : K) - 1);
             } else {
             constexpr int GPC = 32 / NC;        // groups per 32-column chunk
             constexpr int L = 32 / GPC;         // columns per group
@@ -900,7 +1006,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 gm[c * GPC + g] = m;
               }
             }
-            bitonic_desc32(gm);
+            bitonic_desc<32>(gm);
             const int kk = p.k < 32 ? p.k : 32;
             bound = reg_select(gm, kk - 1);
             }
@@ -1006,6 +1112,23 @@ cudaError_t launch_variant(const CUtensorMap& mq, const CUtensorMap& me, const T
   return cudaGetLastError();
 }
 
+// Dual mode (two query tiles per unit); 256-row corpus tiles, lists of 8 or 16.
+template <int K, bool H>
+cudaError_t launch_dual_variant(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
+                                int grid, cudaStream_t st) {
+  constexpr size_t smem = smem_for<256, K, false, true>();
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(tc_search_kernel<256, K, H, false, true>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  tc_search_kernel<256, K, H, false, true><<<grid, threads_for(K), smem, st>>>(mq, me, prm);
+  return cudaGetLastError();
+}
+
 template <int BN, int K>
 cudaError_t launch_k(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm, int grid,
                      bool hybrid, cudaStream_t st) {
@@ -1036,6 +1159,8 @@ cudaError_t launch_pair256_dense(const CUtensorMap& mq, const CUtensorMap& me, c
                                  int grid, cudaStream_t st);
 cudaError_t launch_pair256_fused(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
                                  int grid, cudaStream_t st);
+cudaError_t launch_dual256(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
+                           int grid, bool hybrid, cudaStream_t st);
 
 }  // namespace tc
 }  // namespace oprag

@@ -209,8 +209,9 @@ class Index:
         self.set_option(_lib.OPRAG_OPT_PATH, {None: 0, "simt": 1, "tc": 2}[path])
 
     def force_pair(self, mode: str | None) -> None:
-        """None: automatic; "single": one CTA per MMA; "pair": CTA pairs."""
-        self.set_option(_lib.OPRAG_OPT_PAIR, {None: 0, "single": 1, "pair": 2}[mode])
+        """None: automatic; "single": one CTA per MMA, one query tile per unit;
+        "pair": CTA pairs; "dual": one CTA, two query tiles per unit."""
+        self.set_option(_lib.OPRAG_OPT_PAIR, {None: 0, "single": 1, "pair": 2, "dual": 3}[mode])
 
     def force_block_n(self, bn: int | None) -> None:
         self.set_option(_lib.OPRAG_OPT_BLOCK_N, bn or 0)
@@ -228,11 +229,13 @@ class Index:
     @property
     def last_launch(self) -> dict:
         """Main kernel launch of the last search: grid (CTAs), cluster (2 = CTA
-        pairs), block_n; zeros for the SIMT kernel."""
-        g, c, b = _I32(), _I32(), _I32()
+        pairs), block_n, query tiles per CTA and unit (2 = dual mode); zeros
+        for the SIMT kernel."""
+        g, c, b, t = _I32(), _I32(), _I32(), _I32()
         check(self._lib.oprag_index_last_launch(self._h, ctypes.byref(g), ctypes.byref(c),
                                                 ctypes.byref(b)))
-        return {"grid": g.value, "cluster": c.value, "block_n": b.value}
+        check(self._lib.oprag_index_last_tiles_per_cta(self._h, ctypes.byref(t)))
+        return {"grid": g.value, "cluster": c.value, "block_n": b.value, "tiles": t.value}
 
     @property
     def last_path(self) -> str:

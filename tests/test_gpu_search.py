@@ -240,11 +240,13 @@ def test_shared_bound_tags_wrap_around():
     idx.check()
 
 
-@pytest.mark.parametrize("q,k", [(1024, 5), (1024, 16), (4096, 7), (256, 12)])
+@pytest.mark.parametrize("q,k", [(1024, 5), (1024, 16), (4096, 7), (256, 12),
+                                 (1, 5), (37, 16), (200, 9), (600, 16), (600, 3)])
 def test_merge_regimes(q, k):
     """The final merge runs as one warp per query over at most 32 partial
-    lists (large batches), one warp per query over 33-64 lists, or one CTA
-    per query over more (small batches); all must give the exact top-k."""
+    lists (large batches), one, two or four warps per query over more lists
+    when k <= 16 (by batch size), or one CTA per query for larger k; all
+    must give the exact top-k."""
     rng = np.random.default_rng(q + k)
     n, d = 40000, 256
     E = workloads.to_bf16_bits(workloads._normalise(rng.standard_normal((n, d)).astype(np.float32)))
@@ -252,6 +254,6 @@ def test_merge_regimes(q, k):
     idx = _index(E)
     ids, sc = idx.search(dev_tensor(Q), k)
     assert idx.last_path == "tc"
-    rows = np.sort(rng.choice(q, 40, replace=False))
+    rows = np.sort(rng.choice(q, min(q, 40), replace=False))
     check_dense(ids, sc, E, Q, k, f"merge q={q} k={k}", rows=rows)
     idx.check()
