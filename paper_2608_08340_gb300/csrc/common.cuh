@@ -47,6 +47,15 @@ __device__ __forceinline__ float key_floor(uint64_t k) {
 }
 
 __device__ __forceinline__ uint64_t umax64(uint64_t a, uint64_t b) { return a > b ? a : b; }
+
+// Largest 64-bit key of the warp as two 32-bit warp reductions: the largest
+// high word, then the largest low word among the lanes that hold it.
+__device__ __forceinline__ uint64_t warp_max_key(uint64_t x) {
+  const uint32_t hi = __reduce_max_sync(0xffffffffu, static_cast<uint32_t>(x >> 32));
+  const uint32_t lo = __reduce_max_sync(
+      0xffffffffu, static_cast<uint32_t>(x >> 32) == hi ? static_cast<uint32_t>(x) : 0u);
+  return (static_cast<uint64_t>(hi) << 32) | lo;
+}
 __device__ __forceinline__ uint64_t umin64(uint64_t a, uint64_t b) { return a < b ? a : b; }
 
 // ---------------------------------------------------------------------------

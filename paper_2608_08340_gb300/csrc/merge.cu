@@ -85,9 +85,7 @@ merge_kway_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
   int avail = kHeads;
   uint64_t mine = kEmptyKey;      // the answer of rank (lane + 32 * m) for the current m
   for (int r = 0; r < k; ++r) {
-    uint64_t best = h[0];
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) best = umax64(best, __shfl_xor_sync(0xffffffffu, best, o));
+    const uint64_t best = warp_max_key(h[0]);
     if (best != kEmptyKey && h[0] == best) {
 #pragma unroll
       for (int i = 0; i + 1 < kHeads; ++i) h[i] = h[i + 1];
@@ -171,9 +169,7 @@ merge_small_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
     uint64_t own = key[0][0];
 #pragma unroll
     for (int u = 1; u < kSmallLists; ++u) own = umax64(own, key[u][0]);
-    uint64_t best = own;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) best = umax64(best, __shfl_xor_sync(0xffffffffu, best, o));
+    uint64_t best = warp_max_key(own);
     if constexpr (W > 1) {
       if (lane == 0) heads[r & 1][warp] = best;
       // The query's W warps (named barrier 1 + slot; constant ids, so
