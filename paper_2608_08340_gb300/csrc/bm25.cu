@@ -9,7 +9,8 @@
 // list (a repeated term counts again).
 //
 // One CTA per (query, tile of 8192 chunks) accumulates those sums in shared
-// memory, one term at a time in the query's order.  A dense term (held by
+// memory, one term at a time in the query's order; a table built with the
+// postings gives where each sparse term's postings enter the tile.  A dense term (held by
 // more than half of the chunks, stored as a row of weights with zeros where
 // absent) is added element-wise with 16-byte loads, each thread keeping the
 // same elements, so consecutive dense terms need no barrier; a sparse term
@@ -25,30 +26,12 @@ namespace oprag {
 
 namespace {
 
-constexpr int kDocTile = 8192;
+constexpr int kDocTile = kBm25DocTile;
 constexpr int kBm25Threads = 256;
 constexpr int kTermsPerPass = kBm25Threads / 32;
 constexpr int kScatterUnroll = 4;      // postings loaded per thread before the adds
+constexpr int kDenseBatch = 8;         // dense-row float4 groups loaded per thread before the adds
 constexpr int kSkipTerm = -2;          // term id outside the vocabulary
-
-// First position in [lo, hi) whose chunk is >= key (hi if none); chunks are
-// ascending.  Warp-collective: 32 probes per round.
-__device__ int64_t warp_lower_bound(const int2* a, int64_t lo, int64_t hi, int32_t key) {
-  const int lane = threadIdx.x & 31;
-  while (hi - lo > 32) {
-    const int64_t step = (hi - lo + 31) / 32;
-    const int64_t pos = lo + lane * step;
-    const bool less = pos < hi && a[pos].x < key;
-    const int c = __popc(__ballot_sync(0xffffffffu, less));
-    if (c == 0) return lo;
-    const int64_t next = lo + static_cast<int64_t>(c) * step;
-    lo = lo + static_cast<int64_t>(c - 1) * step + 1;
-    if (c < 32 && next < hi) hi = next;
-  }
-  const int64_t pos = lo + lane;
-  const bool less = pos < hi && a[pos].x < key;
-  return lo + __popc(__ballot_sync(0xffffffffu, less));
-}
 
 __global__ void __launch_bounds__(kBm25Threads)
 bm25_matrix_kernel(SparseIndex sp, int64_t n, const int32_t* __restrict__ q_indptr,
@@ -71,25 +54,25 @@ bm25_matrix_kernel(SparseIndex sp, int64_t n, const int32_t* __restrict__ q_indp
   bool pending = true;      // element-wise work since the last barrier came from a scatter
   for (int base = t0; base < t1; base += kTermsPerPass) {
     // Classify each term of the pass and locate a sparse term's postings
-    // inside [d0, d1): one warp per term.
+    // inside [d0, d1) in the per-tile table: one thread per term, its three
+    // loads issued together.
     const int ti = base + warp;
-    if (ti < t1) {
+    if (ti < t1 && lane == 0) {
       const int32_t term = q_terms[ti];
       int slot = kSkipTerm;
       int64_t lo = 0, hi = 0;
       if (term >= 0 && term < sp.vocab) {
+        const int64_t* tp = sp.tile_ptr + static_cast<int64_t>(term) * (sp.ntiles + 1) + blockIdx.y;
+        const int64_t a = tp[0], z = tp[1];
         slot = sp.dense_slot[term];
         if (slot < 0) {
-          const int64_t p0 = sp.post_ptr[term], p1 = sp.post_ptr[term + 1];
-          lo = warp_lower_bound(sp.post, p0, p1, static_cast<int32_t>(d0));
-          hi = warp_lower_bound(sp.post, lo, p1, static_cast<int32_t>(d1));
+          lo = a;
+          hi = z;
         }
       }
-      if (lane == 0) {
-        slot_of[warp] = slot;
-        rng_lo[warp] = lo;
-        rng_hi[warp] = hi;
-      }
+      slot_of[warp] = slot;
+      rng_lo[warp] = lo;
+      rng_hi[warp] = hi;
     }
     __syncthreads();
     pending = false;
@@ -102,15 +85,28 @@ bm25_matrix_kernel(SparseIndex sp, int64_t n, const int32_t* __restrict__ q_indp
         // Dense term: thread i owns float4 groups i, i + 256, ...; after
         // another dense term nothing needs ordering.
         if (pending) __syncthreads();
+        // The row's groups are loaded kDenseBatch at a time, all before the
+        // adds, so a dense term costs one L2 round trip per batch.
         const float4* row = reinterpret_cast<const float4*>(sp.dense_w + slot * sp.dense_ld + d0);
-        for (int i = threadIdx.x; i < nv; i += blockDim.x) {
-          const float4 x = __ldg(row + i);
-          float4 a = acc4[i];
-          a.x += x.x;
-          a.y += x.y;
-          a.z += x.z;
-          a.w += x.w;
-          acc4[i] = a;
+        for (int i0 = threadIdx.x; i0 < nv; i0 += kDenseBatch * kBm25Threads) {
+          float4 x[kDenseBatch];
+#pragma unroll
+          for (int u = 0; u < kDenseBatch; ++u) {
+            const int i = i0 + u * kBm25Threads;
+            x[u] = i < nv ? __ldg(row + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+          }
+#pragma unroll
+          for (int u = 0; u < kDenseBatch; ++u) {
+            const int i = i0 + u * kBm25Threads;
+            if (i < nv) {
+              float4 a = acc4[i];
+              a.x += x[u].x;
+              a.y += x[u].y;
+              a.z += x[u].z;
+              a.w += x[u].w;
+              acc4[i] = a;
+            }
+          }
         }
         pending = false;
         dirty = true;

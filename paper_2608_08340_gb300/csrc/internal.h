@@ -124,6 +124,9 @@ cudaError_t launch_merge_two(int q, const int64_t* a_ids, const float* a_sc, int
 // Terms held by more than half of the chunks are stored as dense rows of
 // w(t, .) (zero where absent: 4 bytes per chunk instead of 8 per posting, and
 // no scatter); the other terms as postings.
+// Chunks per tile of the BM25 pass (one CTA per query and tile).
+constexpr int kBm25DocTile = 8192;
+
 struct SparseIndex {
   int vocab;
   int64_t nnz;               // postings of the sparse terms
@@ -132,6 +135,10 @@ struct SparseIndex {
   const int32_t* dense_slot; // device, vocab: row of a dense term, -1 otherwise
   const float* dense_w;      // device, rows x dense_ld
   int64_t dense_ld;          // multiple of 4, >= n; zero past n
+  // device, vocab x (ntiles + 1): entry (t, b) is the first posting of term t
+  // whose chunk is >= b * kBm25DocTile (post_ptr[t + 1] past the last).
+  const int64_t* tile_ptr;
+  int ntiles;
 };
 cudaError_t launch_bm25_matrix(const SparseIndex& sp, int64_t n, const int32_t* q_indptr,
                                const int32_t* q_terms, int q, float* out, int64_t ld,

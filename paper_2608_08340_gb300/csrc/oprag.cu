@@ -94,6 +94,8 @@ struct oprag_index {
   int32_t* dense_slot = nullptr;
   float* dense_w = nullptr;
   int64_t dense_ld = 0;
+  int64_t* tile_ptr = nullptr;
+  int ntiles = 0;
 
   int opt_path = 0;
   int opt_block_n = 0;
@@ -158,10 +160,12 @@ struct oprag_index {
     if (post) cudaFree(post);
     if (dense_slot) cudaFree(dense_slot);
     if (dense_w) cudaFree(dense_w);
+    if (tile_ptr) cudaFree(tile_ptr);
     post_ptr = nullptr;
     post = nullptr;
     dense_slot = nullptr;
     dense_w = nullptr;
+    tile_ptr = nullptr;
     has_sparse = false;
   }
 };
@@ -806,6 +810,18 @@ int rebuild_sparse(oprag_index* idx) {
       post[fill[t]++] = make_int2(dd, bits);
     }
   }
+  // Where each term's postings enter each tile of the BM25 pass.
+  const int ntiles = static_cast<int>((n + kBm25DocTile - 1) / kBm25DocTile);
+  std::vector<int64_t> tptr(static_cast<size_t>(vocab) * (ntiles + 1));
+  for (int t = 0; t < vocab; ++t) {
+    int64_t* row = tptr.data() + static_cast<size_t>(t) * (ntiles + 1);
+    int64_t p = ptr[t];
+    for (int tb = 0; tb <= ntiles; ++tb) {
+      const int64_t doc0 = static_cast<int64_t>(tb) * kBm25DocTile;
+      while (p < ptr[t + 1] && post[p].x < doc0) ++p;
+      row[tb] = p;
+    }
+  }
 
   DeviceGuard g(idx->device);
   cudaError_t e = idx->drain();
@@ -815,7 +831,8 @@ int rebuild_sparse(oprag_index* idx) {
   if (cudaMalloc(&idx->post_ptr, ptr.size() * sizeof(int64_t)) != cudaSuccess ||
       cudaMalloc(&idx->post, std::max<int64_t>(nnz, 1) * sizeof(int2)) != cudaSuccess ||
       cudaMalloc(&idx->dense_slot, slot.size() * sizeof(int32_t)) != cudaSuccess ||
-      cudaMalloc(&idx->dense_w, std::max<size_t>(dense.size(), 4) * sizeof(float)) != cudaSuccess) {
+      cudaMalloc(&idx->dense_w, std::max<size_t>(dense.size(), 4) * sizeof(float)) != cudaSuccess ||
+      cudaMalloc(&idx->tile_ptr, tptr.size() * sizeof(int64_t)) != cudaSuccess) {
     cudaGetLastError();
     idx->free_sparse();
     return fail(OPRAG_ERR_OOM, "cannot allocate postings");
@@ -827,12 +844,15 @@ int rebuild_sparse(oprag_index* idx) {
     e = cudaMemcpy(idx->dense_slot, slot.data(), slot.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
   if (e == cudaSuccess && !dense.empty())
     e = cudaMemcpy(idx->dense_w, dense.data(), dense.size() * sizeof(float), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(idx->tile_ptr, tptr.data(), tptr.size() * sizeof(int64_t), cudaMemcpyHostToDevice);
   if (e != cudaSuccess) {
     idx->free_sparse();
     return cuda_fail(e, "uploading postings");
   }
   idx->nnz = nnz;
   idx->dense_ld = dld;
+  idx->ntiles = ntiles;
   idx->has_sparse = true;
   return ok();
 }
@@ -920,7 +940,8 @@ int oprag_hybrid_search(oprag_index* idx, const void* queries, int32_t q, const 
     return rc;
   if ((rc = begin_call(idx, st))) return rc;
   const SparseIndex sp{idx->vocab,      idx->nnz,     idx->post_ptr, idx->post,
-                       idx->dense_slot, idx->dense_w, idx->dense_ld};
+                       idx->dense_slot, idx->dense_w, idx->dense_ld, idx->tile_ptr,
+                       idx->ntiles};
   const size_t qrow = static_cast<size_t>(idx->d) * elem_size(idx->dtype);
   for (int c0 = 0; c0 < q; c0 += qchunk) {
     const int qc = std::min(qchunk, q - c0);
@@ -967,7 +988,8 @@ int oprag_hybrid_search_dense_first(oprag_index* idx, const void* queries, int32
   const Fusion none{nullptr, 0, nullptr, 0.f};
   if ((rc = run_search(idx, queries, q, nc, none, cid, csc, st))) return rc;
   const SparseIndex sp{idx->vocab,      idx->nnz,     idx->post_ptr, idx->post,
-                       idx->dense_slot, idx->dense_w, idx->dense_ld};
+                       idx->dense_slot, idx->dense_w, idx->dense_ld, idx->tile_ptr,
+                       idx->ntiles};
   cudaError_t e = launch_rerank(sp, q, nc, cid, csc, q_indptr, q_terms, alpha, k, out_ids,
                                 out_scores, st);
   if (e != cudaSuccess) return cuda_fail(e, "rerank kernel");
