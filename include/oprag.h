@@ -253,8 +253,8 @@ OPRAG_API int oprag_index_set_option(oprag_index *idx, int32_t option, int32_t v
  * 256-row corpus tiles; ignored with 128-row tiles).  1 runs every CTA on its
  * own (M = 128 MMAs), one query tile per unit.  3 (dual mode) runs every CTA
  * on its own with two query tiles per unit that share each corpus tile
- * (256-row tiles; k <= 16 and more than 128 queries, ignored otherwise).
- * 0 (default) chooses dual mode when its units fit in one wave of CTAs,
+ * (128-row tiles; k <= 16 and more than 128 queries, ignored otherwise).
+ * 0 (default) chooses dual mode when its units come to at most two per CTA,
  * single CTAs otherwise. */
 #define OPRAG_OPT_PAIR 4
 

@@ -64,17 +64,17 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
     const int64_t units256 = static_cast<int64_t>(pl.qt) * ((s.n + 255) / 256);
     if (units256 < 4LL * num_sms) bn = 128;
   }
-  // Dual mode: every unit takes two query tiles and one 256-row corpus tile,
-  // so a CTA reads each corpus tile once for 256 queries.  Automatic when
-  // there are at least two query tiles and the dual units fit in one wave
-  // (small batches, where the copies into the SMs, not the MMAs, bound the
-  // kernel and no unit's epilogue has a next unit to overlap); it needs the
-  // two epilogue sets of lists of 8 or 16.
+  // Dual mode: every unit takes two query tiles and one 128-row corpus tile,
+  // so a CTA reads each corpus tile once for 256 queries, and its four
+  // accumulators let one unit's epilogue overlap the next unit.  Automatic
+  // when there are at least two query tiles and at most two dual units per
+  // CTA (small batches, where the copies into the SMs, not the MMAs, bound
+  // the kernel); it needs the two epilogue sets of lists of 8 or 16.
   const bool dual_ok = pl.qt >= 2 && epi_sets(list_len_for(s.k)) == 2 && force_pair != 2 &&
-                       (force_block_n == 0 || force_block_n == 256);
-  const int64_t dual_units = static_cast<int64_t>((pl.qt + 1) / 2) * ((s.n + 255) / 256);
-  pl.dual = dual_ok && (force_pair == 3 || (force_pair == 0 && dual_units <= num_sms));
-  if (pl.dual) bn = 256;
+                       (force_block_n == 0 || force_block_n == 128);
+  const int64_t dual_units = static_cast<int64_t>((pl.qt + 1) / 2) * ((s.n + 127) / 128);
+  pl.dual = dual_ok && (force_pair == 3 || (force_pair == 0 && dual_units <= 2LL * num_sms));
+  if (pl.dual) bn = 128;
   pl.block_n = bn;
   // CTA pairs cut the operand bytes each SM loads per MMA by a third; they
   // need 256-row corpus tiles and a device that fits clusters of two.  They
@@ -129,7 +129,7 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
   const size_t b_stage = static_cast<size_t>(pair ? bn / 2 : bn) * 128;
   const size_t a_stage = kAStageBytes * (pl.dual ? 2 : 1);
   pl.stages = pair      ? stages_for<256, true>()
-              : pl.dual ? stages_for<256, false, true>()
+              : pl.dual ? stages_for<128, false, true>()
                         : (bn == 128 ? stages_for<128>() : stages_for<256>());
   pl.smem = static_cast<size_t>(pl.stages) * (a_stage + b_stage) +
             static_cast<size_t>(epi_sets(K)) * 128 * kStageRowBytes + 1024 + 256;
@@ -203,8 +203,8 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
   lists->pair = pl.dual ? 2 : pl.pair;
   const bool hybrid = fu.bm25 != nullptr;
   if (pl.dual) {
-    if (pl.block_n != 256) return cudaErrorInvalidValue;
-    return launch_dual256(mq, me, prm, pl.grid, hybrid, st);
+    if (pl.block_n != 128) return cudaErrorInvalidValue;
+    return launch_dual128(mq, me, prm, pl.grid, hybrid, st);
   }
   if (pl.pair == 2) {
     if (pl.block_n != 256) return cudaErrorInvalidValue;

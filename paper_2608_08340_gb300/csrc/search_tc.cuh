@@ -586,22 +586,25 @@ struct EpiList<K, true> {
 // 128 x 16 + BN x 16.  The unit sequence (UnitSeq) runs over pairs: p.qt
 // counts pairs of query tiles and the pair index plays the CTA index.
 //
-// kDual: every unit covers query tiles 2J and 2J + 1 and corpus tile t; a
-// stage holds both query tiles' K-block and the corpus tile's, and the MMA
-// warp issues two MMAs per K-step that share the corpus operand, one into
-// each accumulator.  Epilogue set s filters query tile 2J + s.  Per unit the
-// CTA reads the corpus tile once for 256 queries, so small batches (one unit
-// per CTA) load half the operand bytes of two single-tile units.
+// kDual (BN = 128): every unit covers query tiles 2J and 2J + 1 and corpus
+// tile t; a stage holds both query tiles' K-block and the corpus tile's, and
+// the MMA warp issues two MMAs per K-step that share the corpus operand, one
+// into each accumulator of the unit's buffer (four accumulators of BN
+// columns: buffer u & 1, query tile s at column (2 (u & 1) + s) BN).
+// Epilogue set s filters query tile 2J + s, so one unit's epilogue overlaps
+// the next unit's copies and MMAs.  Per unit the CTA reads the corpus tile
+// once for 256 queries.
 template <int BN, int K, bool kHybrid, bool kPair = false, bool kDual = false>
 __global__ void __launch_bounds__(threads_for(K), 1)
 tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_e,
                  const TcParams p) {
   static_assert(!(kPair && kDual), "pair and dual modes are exclusive");
   static_assert(!kDual || epi_sets(K) == 2, "dual mode needs one epilogue set per query tile");
+  static_assert(!kDual || BN == 128, "dual mode double-buffers four accumulators of 128 columns");
   constexpr int S = stages_for<BN, kPair, kDual>();
   constexpr uint32_t kAStage = a_stage_bytes<kDual>();
   constexpr uint32_t kBStageBytes = b_stage_bytes<BN, kPair>();
-  constexpr uint32_t kTmemCols = 2 * BN;
+  constexpr uint32_t kTmemCols = (kDual ? 4 : 2) * BN;
   constexpr int kEpiSets = epi_sets(K);
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* base = reinterpret_cast<unsigned char*>(
@@ -612,8 +615,8 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
   uint64_t* full = reinterpret_cast<uint64_t*>(stage_rows + kEpiSets * 128 * 32);
   uint64_t* empty = full + S;
   uint64_t* tfull = empty + S;
-  uint64_t* tempty = tfull + 2;
-  uint64_t* mma_done = tempty + 2;
+  uint64_t* tempty = tfull + 4;
+  uint64_t* mma_done = tempty + 4;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
@@ -639,7 +642,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < 4; ++b) {     // accumulators 2 and 3: dual mode only
       mbar_init(&tfull[b], 1);
       mbar_init(&tempty[b], kPair ? 8 : 4);   // four epilogue warps per CTA
     }
@@ -735,10 +738,13 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       UnitSeq us;
       for (us.start(p, cta, C); ok && us.valid(); us.next()) {
         if constexpr (kDual) {
-          // Both accumulators take this unit.
-          if (!mbar_wait(&tempty[0], acc_ph ^ 1u, abort_flag, p.dev_err)) break;
-          if (!mbar_wait(&tempty[1], acc_ph ^ 1u, abort_flag, p.dev_err)) break;
+          // Both accumulators of buffer acc take this unit.
+          const int a0i = 2 * acc, a1i = 2 * acc + 1;
+          if (!mbar_wait(&tempty[a0i], acc_ph ^ 1u, abort_flag, p.dev_err)) break;
+          if (!mbar_wait(&tempty[a1i], acc_ph ^ 1u, abort_flag, p.dev_err)) break;
           tc_fence_after();
+          const uint32_t d0 = tmem_base + static_cast<uint32_t>(a0i * BN);
+          const uint32_t d1 = tmem_base + static_cast<uint32_t>(a1i * BN);
           for (int kb = 0; kb < p.kblocks; ++kb) {
             if (!mbar_wait(&full[s], ph, abort_flag, p.dev_err)) { ok = false; break; }
             tc_fence_after();
@@ -748,16 +754,16 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
 #pragma unroll
             for (int kk = 0; kk < kBlockK / kUmmaK; ++kk) {
               const uint32_t accum = (kb | kk) != 0 ? 1u : 0u;
-              mma_bf16(tmem_base, a0 + 2 * kk, b + 2 * kk, idesc, accum);
-              mma_bf16(tmem_base + static_cast<uint32_t>(BN), a1 + 2 * kk, b + 2 * kk, idesc, accum);
+              mma_bf16(d0, a0 + 2 * kk, b + 2 * kk, idesc, accum);
+              mma_bf16(d1, a1 + 2 * kk, b + 2 * kk, idesc, accum);
             }
             mma_commit(&empty[s]);
             if (++s == S) { s = 0; ph ^= 1u; }
           }
           if (!ok) break;
-          mma_commit(&tfull[0]);
-          mma_commit(&tfull[1]);
-          acc_ph ^= 1u;
+          mma_commit(&tfull[a0i]);
+          mma_commit(&tfull[a1i]);
+          if (++acc == 2) { acc = 0; acc_ph ^= 1u; }
           continue;
         }
         if (!mbar_wait<kPair>(&tempty[acc], acc_ph ^ 1u, abort_flag, p.dev_err)) break;
@@ -828,12 +834,13 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     int cur_j = -1;
     int64_t cur_sr = 0;
     bool cur_valid = false;
-    uint32_t acc_ph = 0;                     // phase bit per accumulator
+    uint32_t acc_ph = 0;                     // phase bit per accumulator (bit acc)
     UnitSeq us;
     int seq = 0;
     for (us.start(p, cta, C); us.valid(); us.next(), ++seq) {
       if (!kDual && seq % kEpiSets != set) continue;
-      const int acc = kDual ? set : (seq & 1);
+      // Accumulator (TMEM columns acc * BN, barriers tfull / tempty [acc]).
+      const int acc = kDual ? 2 * (seq & 1) + set : (seq & 1);
       const int J = us.j();
       const int j = qtile(J);                // this CTA's query tile
       const int64_t t = us.t();
@@ -1112,20 +1119,20 @@ cudaError_t launch_variant(const CUtensorMap& mq, const CUtensorMap& me, const T
   return cudaGetLastError();
 }
 
-// Dual mode (two query tiles per unit); 256-row corpus tiles, lists of 8 or 16.
+// Dual mode (two query tiles per unit); 128-row corpus tiles, lists of 8 or 16.
 template <int K, bool H>
 cudaError_t launch_dual_variant(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
                                 int grid, cudaStream_t st) {
-  constexpr size_t smem = smem_for<256, K, false, true>();
+  constexpr size_t smem = smem_for<128, K, false, true>();
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(tc_search_kernel<256, K, H, false, true>,
+    cudaError_t e = cudaFuncSetAttribute(tc_search_kernel<128, K, H, false, true>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  tc_search_kernel<256, K, H, false, true><<<grid, threads_for(K), smem, st>>>(mq, me, prm);
+  tc_search_kernel<128, K, H, false, true><<<grid, threads_for(K), smem, st>>>(mq, me, prm);
   return cudaGetLastError();
 }
 
@@ -1159,7 +1166,7 @@ cudaError_t launch_pair256_dense(const CUtensorMap& mq, const CUtensorMap& me, c
                                  int grid, cudaStream_t st);
 cudaError_t launch_pair256_fused(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
                                  int grid, cudaStream_t st);
-cudaError_t launch_dual256(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
+cudaError_t launch_dual128(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
                            int grid, bool hybrid, cudaStream_t st);
 
 }  // namespace tc

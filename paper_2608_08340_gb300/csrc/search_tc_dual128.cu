@@ -1,11 +1,11 @@
 // Tensor-core search kernels in dual mode (two query tiles per unit,
-// 256-row corpus tiles; lists of 8 or 16 keys).
+// 128-row corpus tiles, double-buffered accumulators; lists of 8 or 16 keys).
 #include "search_tc.cuh"
 
 namespace oprag {
 namespace tc {
 
-cudaError_t launch_dual256(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
+cudaError_t launch_dual128(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
                            int grid, bool hybrid, cudaStream_t st) {
   switch (list_len_for(prm.k)) {
     case 8:

@@ -33,12 +33,12 @@ def _search(idx, Q, k, mode):
     assert launch["cluster"] == 1, launch
     assert launch["tiles"] == (2 if mode == "dual" else 1), launch
     if mode == "dual":
-        assert launch["block_n"] == 256, launch
+        assert launch["block_n"] == 128, launch
     return out
 
 
 @pytest.mark.parametrize("n,d,q,k", [
-    (32768, 768, 256, 5),      # the paper-shaped small batch: one unit per CTA
+    (32768, 768, 256, 5),      # the paper-shaped small batch: one or two units per CTA
     (9000, 768, 300, 10),      # three query tiles: the second unit's second tile ragged
     (5000, 128, 257, 1),       # three tiles, the third holds one query
     (4097, 136, 129, 5),       # two tiles, the second holds one query; ragged d and n
