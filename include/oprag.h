@@ -254,7 +254,7 @@ OPRAG_API int oprag_index_set_option(oprag_index *idx, int32_t option, int32_t v
  * own (M = 128 MMAs), one query tile per unit.  3 (dual mode) runs every CTA
  * on its own with two query tiles per unit that share each corpus tile
  * (128-row tiles; k <= 16 and more than 128 queries, ignored otherwise).
- * 0 (default) chooses dual mode when its units come to at most two per CTA,
+ * 0 (default) chooses dual mode when its units come to at most four per CTA,
  * single CTAs otherwise. */
 #define OPRAG_OPT_PAIR 4
 

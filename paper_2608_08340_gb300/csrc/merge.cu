@@ -5,7 +5,7 @@
 // are corpus slices instead of index shards.
 //
 // Three merges by list count and k: one warp per query over at most 32
-// sorted lists (head by head), one to four warps per query over up to 384
+// sorted lists (head by head), one to four warps per query over up to 512
 // lists when k <= 16 (also head by head), and the block merge of merge.cuh
 // (one CTA per query) otherwise.
 #include "merge.cuh"
@@ -125,7 +125,7 @@ merge_kway_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
 // next keys once the held ones are used up, which only k > kSmallKeys can
 // need).
 constexpr int kSmallThreads = 128;
-constexpr int kSmallLists = 3;
+constexpr int kSmallLists = 4;
 constexpr int kSmallKeys = 6;
 
 template <int W>

@@ -67,13 +67,14 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
   // Dual mode: every unit takes two query tiles and one 128-row corpus tile,
   // so a CTA reads each corpus tile once for 256 queries, and its four
   // accumulators let one unit's epilogue overlap the next unit.  Automatic
-  // when there are at least two query tiles and at most two dual units per
+  // when there are at least two query tiles and at most four dual units per
   // CTA (small batches, where the copies into the SMs, not the MMAs, bound
-  // the kernel); it needs the two epilogue sets of lists of 8 or 16.
+  // the kernel; measured on 32768 x 768: faster up to 512 queries, slower at
+  // 1024); it needs the two epilogue sets of lists of 8 or 16.
   const bool dual_ok = pl.qt >= 2 && epi_sets(list_len_for(s.k)) == 2 && force_pair != 2 &&
                        (force_block_n == 0 || force_block_n == 128);
   const int64_t dual_units = static_cast<int64_t>((pl.qt + 1) / 2) * ((s.n + 127) / 128);
-  pl.dual = dual_ok && (force_pair == 3 || (force_pair == 0 && dual_units <= 2LL * num_sms));
+  pl.dual = dual_ok && (force_pair == 3 || (force_pair == 0 && dual_units <= 4LL * num_sms));
   if (pl.dual) bn = 128;
   pl.block_n = bn;
   // CTA pairs cut the operand bytes each SM loads per MMA by a third; they
