@@ -113,7 +113,8 @@ merge_kway_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
 }
 
 // More than 32 lists and k <= 16, at most kSmallLists lists per lane: W
-// warps per query (W = 4, 2 or 1; CTAs of four warps, 4 / W queries each).
+// warps per query (W = 1, 2 or 4 by list count; CTAs of four warps, 4 / W
+// queries each).
 // Launched early (programmatic dependent
 // launch), a CTA waits in place and starts as soon as the search grid ends.
 // Lane l of warp w holds lists p = 32 w + l + 32 W u (u < kSmallLists): the
@@ -245,18 +246,16 @@ cudaError_t launch_small_w(const ListSet& ls, int q, int k, int64_t* out_ids, fl
                             levels_out);
 }
 
-// Warps per query of merge_small_kernel: four while one merge CTA per SM
-// covers the batch, else two, else one.  Returns cudaErrorNotSupported when
-// a lane would hold more than kSmallLists lists (the caller then takes the
-// block merge).
+// Warps per query of merge_small_kernel: the fewest whose lanes hold all of
+// a query's lists (kSmallLists each).  The lists' loads are issued together
+// whatever W is, and with one warp per query the head-by-head rounds need no
+// barrier.  Returns cudaErrorNotSupported when four warps do not suffice (the
+// caller then takes the block merge).
 cudaError_t launch_small(const ListSet& ls, int q, int k, int64_t* out_ids, float* out_scores,
                          cudaStream_t st, float* kth_out, float* levels_out) {
-  int dev = 0, sms = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-    sms = 1;
-  const int W = q <= sms ? 4 : q <= 2 * sms ? 2 : 1;
-  if (ls.P > kSmallLists * 32 * W) return cudaErrorNotSupported;
+  constexpr int kPerWarp = kSmallLists * 32;
+  const int W = ls.P <= kPerWarp ? 1 : ls.P <= 2 * kPerWarp ? 2 : 4;
+  if (ls.P > W * kPerWarp) return cudaErrorNotSupported;
   if (W == 4) return launch_small_w<4>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
   if (W == 2) return launch_small_w<2>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
   return launch_small_w<1>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);

@@ -7,7 +7,6 @@
 #include <cstring>
 #include <mutex>
 #include <string>
-#include <unordered_set>
 #include <vector>
 
 #include "oprag.h"
@@ -514,17 +513,25 @@ int oprag_upsert(oprag_index* idx, const int64_t* ids, const void* rows, int64_t
                   (long long)ids[i], (long long)idx->n);
   if (rows_on_device && (reinterpret_cast<uintptr_t>(rows) & 15))
     return fail(OPRAG_ERR_INVALID_ARG, "device rows must be 16-byte aligned");
-  // The later entry of a repeated id wins: keep the last occurrence only.
+  // The later entry of a repeated id wins: keep the last occurrence only
+  // (walking backwards through an open-addressing set of the ids seen, at
+  // most half full).
   std::vector<int64_t> pairs;
   pairs.reserve(2 * m);
   {
-    std::unordered_set<int64_t> seen;
-    seen.reserve(static_cast<size_t>(m) * 2);
-    for (int64_t i = m - 1; i >= 0; --i)
-      if (seen.insert(ids[i]).second) {
-        pairs.push_back(i);
-        pairs.push_back(ids[i]);
-      }
+    size_t cap = 16;
+    while (cap < static_cast<size_t>(m) * 2) cap <<= 1;
+    std::vector<int64_t> seen(cap, -1);
+    const size_t mask = cap - 1;
+    for (int64_t i = m - 1; i >= 0; --i) {
+      const int64_t id = ids[i];
+      size_t h = (static_cast<uint64_t>(id) * 0x9E3779B97F4A7C15ull) >> 20 & mask;
+      while (seen[h] != -1 && seen[h] != id) h = (h + 1) & mask;
+      if (seen[h] == id) continue;
+      seen[h] = id;
+      pairs.push_back(i);
+      pairs.push_back(id);
+    }
   }
   const int64_t count = static_cast<int64_t>(pairs.size() / 2);
   DeviceGuard g(idx->device);
