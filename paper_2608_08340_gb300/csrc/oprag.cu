@@ -70,6 +70,7 @@ struct oprag_index {
   int dtype = OPRAG_BF16;
   void* emb = nullptr;
   int* dev_err = nullptr;
+  int* err_host = nullptr;       // pinned copy of dev_err, read after host-buffer calls
   cudaEvent_t done = nullptr;
 
   void* scratch = nullptr;     // partial top-k lists
@@ -386,6 +387,12 @@ int oprag_index_create(oprag_index** out, const void* emb, int64_t n, int32_t d,
     idx->dev_err = nullptr;
     return bail(fail(OPRAG_ERR_OOM, "cannot allocate the error word"));
   }
+  if (cudaMallocHost(reinterpret_cast<void**>(&idx->err_host), sizeof(int)) != cudaSuccess) {
+    cudaGetLastError();
+    idx->err_host = nullptr;
+    return bail(fail(OPRAG_ERR_OOM, "cannot allocate the pinned error word"));
+  }
+  *idx->err_host = 0;
   if ((e = cudaEventCreateWithFlags(&idx->done, cudaEventDisableTiming)) != cudaSuccess)
     return bail(cuda_fail(e, "event"));
   cudaStream_t st;
@@ -428,6 +435,7 @@ void oprag_index_destroy(oprag_index* idx) {
   idx->drain();
   if (idx->emb) cudaFree(idx->emb);
   if (idx->dev_err) cudaFree(idx->dev_err);
+  if (idx->err_host) cudaFreeHost(idx->err_host);
   if (idx->gcache.exec) cudaGraphExecDestroy(idx->gcache.exec);
   if (idx->scratch) cudaFree(idx->scratch);
   if (idx->qfloor) cudaFree(idx->qfloor);
@@ -748,10 +756,14 @@ int oprag_search_host(oprag_index* idx, const void* queries, int32_t q, int32_t 
   if (e == cudaSuccess)
     e = cudaMemcpyAsync(out_scores, stage + sc_off, static_cast<size_t>(q) * k * sizeof(float),
                         cudaMemcpyDeviceToHost, st);
+  // The error word travels with the results, so that the call waits for the
+  // device once.
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(idx->err_host, idx->dev_err, sizeof(int), cudaMemcpyDeviceToHost, st);
   if (e != cudaSuccess) return cuda_fail(e, "copying results");
   if ((rc = end_call(idx, st))) return rc;
   if ((e = cudaStreamSynchronize(st)) != cudaSuccess) return cuda_fail(e, "search");
-  return oprag_index_check(idx);
+  return *idx->err_host != 0 ? oprag_index_check(idx) : ok();
 }
 
 // Builds the device side of BM25 (per-posting weights, dense rows of the
