@@ -255,7 +255,8 @@ OPRAG_API int oprag_index_set_option(oprag_index *idx, int32_t option, int32_t v
  * on its own with two query tiles per unit that share each corpus tile
  * (128-row tiles; k <= 16 and more than 128 queries, ignored otherwise).
  * 0 (default) chooses dual mode when its units come to at most four per CTA,
- * single CTAs otherwise. */
+ * CTA pairs for k > 32 with at least 1024 queries on 256-row tiles, single
+ * CTAs otherwise. */
 #define OPRAG_OPT_PAIR 4
 
 /* OPRAG_OPT_BOUND_TAG (test hook): sets the 32-bit tag of the last search's

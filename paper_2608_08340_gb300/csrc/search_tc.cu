@@ -79,10 +79,13 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
   pl.block_n = bn;
   // CTA pairs cut the operand bytes each SM loads per MMA by a third; they
   // need 256-row corpus tiles and a device that fits clusters of two.  They
-  // run only on request: measured on GB300 they are no faster than single
-  // CTAs (the stage rate is the same; the epilogue and the copy/MMA overlap,
-  // not operand bytes, bound the kernel).
-  const bool pair = bn == 256 && pair_capacity > 0 && force_pair == 2;
+  // run on request, and by default for large batches with buffered lists
+  // (k > 32, at least 8 query tiles): measured on GB300, 1M x 768 with 2048
+  // queries and k = 100 takes 2524 instead of 2591 us; with lists of 16
+  // (32768 x 1024, 4096 queries, k = 10) pairs are no faster.
+  const bool pair = bn == 256 && pair_capacity > 0 &&
+                    (force_pair == 2 ||
+                     (force_pair == 0 && list_len_for(s.k) > 32 && pl.qt >= 8));
   pl.pair = pair ? 2 : 1;
   pl.uqt = pair || pl.dual ? (pl.qt + 1) / 2 : pl.qt;
   pl.tile_stride = tile_stride < 1 ? 1 : tile_stride;
