@@ -305,6 +305,22 @@ OPRAG_API int oprag_index_last_launch(const oprag_index *idx, int32_t *grid, int
  * 0 for the SIMT kernel.  OPRAG_ERR_NOT_READY before the first search. */
 OPRAG_API int oprag_index_last_tiles_per_cta(const oprag_index *idx, int32_t *tiles);
 
+/* Host-side plan of a tensor-core search of q queries of dimension d over n
+ * chunks with k results (bf16 index), for a device of num_sms SMs, without
+ * any device work (usable without a GPU).  force_block_n (0, 128, 256) and
+ * force_pair (0 automatic, 1 single CTAs, 2 CTA pairs, 3 dual mode) mean what
+ * OPRAG_OPT_BLOCK_N and OPRAG_OPT_PAIR mean; pair_capacity is the number of
+ * two-CTA clusters the device fits at once (0: no pair mode).  out[0..12]
+ * receives, in order: CTAs launched, corpus rows per tile, CTAs per cluster
+ * (1 or 2), dual mode (0 or 1), query tiles, query tiles of the schedule,
+ * corpus tiles, corpus tiles per L2 window, list slots per query tile,
+ * pipeline stages, dynamic shared memory per CTA in bytes, list scratch in
+ * bytes, and list slots per producer and query tile.  OPRAG_ERR_INVALID_ARG
+ * for n, d, q, k or num_sms < 1, d % 8 != 0, k > OPRAG_K_MAX, or a NULL out. */
+OPRAG_API int oprag_plan_search(int64_t n, int32_t d, int32_t q, int32_t k, int32_t num_sms,
+                                int32_t force_block_n, int32_t force_pair,
+                                int32_t pair_capacity, int64_t *out);
+
 /*
  * oprag_search without any device allocation.  The paper has no counterpart:
  * this entry point serves callers that must not allocate device memory while

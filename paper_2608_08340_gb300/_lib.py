@@ -59,6 +59,8 @@ SIGNATURES = {
     "oprag_index_last_launch": (_I32, [_P, ctypes.POINTER(_I32), ctypes.POINTER(_I32),
                                        ctypes.POINTER(_I32)]),
     "oprag_index_last_tiles_per_cta": (_I32, [_P, ctypes.POINTER(_I32)]),
+    "oprag_plan_search": (_I32, [ctypes.c_int64, _I32, _I32, _I32, _I32, _I32, _I32, _I32,
+                                 ctypes.POINTER(ctypes.c_int64)]),
     "oprag_index_last_timing": (_I32, [_P, ctypes.POINTER(_F), ctypes.POINTER(_F),
                                        ctypes.POINTER(_F)]),
     "oprag_last_error": (ctypes.c_char_p, []),

@@ -1108,6 +1108,25 @@ int oprag_index_last_launch(const oprag_index* idx, int32_t* grid, int32_t* clus
   return ok();
 }
 
+int oprag_plan_search(int64_t n, int32_t d, int32_t q, int32_t k, int32_t num_sms,
+                      int32_t force_block_n, int32_t force_pair, int32_t pair_capacity,
+                      int64_t* out) {
+  if (!out) return fail(OPRAG_ERR_INVALID_ARG, "NULL out");
+  if (n < 1 || d < 1 || q < 1 || k < 1 || num_sms < 1 || d % 8 != 0 || k > OPRAG_K_MAX)
+    return fail(OPRAG_ERR_INVALID_ARG, "bad plan shape n=%lld d=%d q=%d k=%d sms=%d",
+                (long long)n, d, q, k, num_sms);
+  const SearchShape s{n, d, q, k};
+  const TcPlan pl = tc_plan(s, num_sms, force_block_n, 1, force_pair, pair_capacity);
+  const int K = list_len_for(k);
+  const int64_t v[13] = {pl.grid,  pl.block_n, pl.pair,  pl.dual ? 1 : 0,
+                         pl.qt,    pl.uqt,     pl.nt,    pl.win,
+                         pl.pmax,  pl.stages,  static_cast<int64_t>(pl.smem),
+                         static_cast<int64_t>(tc_scratch_bytes(s, pl)),
+                         pl.dual ? 1 : (K <= 16 ? 2 : 1)};
+  for (int i = 0; i < 13; ++i) out[i] = v[i];
+  return ok();
+}
+
 int oprag_index_last_tiles_per_cta(const oprag_index* idx, int32_t* tiles) {
   if (!idx) return fail(OPRAG_ERR_INVALID_ARG, "index is NULL");
   if (!idx->last_path) return fail(OPRAG_ERR_NOT_READY, "no search was issued");

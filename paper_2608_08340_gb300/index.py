@@ -277,3 +277,17 @@ def search_two(knowledge: Index, memory: Index, queries: torch.Tensor, k: int, s
                                           _ptr(src), _ptr(scores), _stream_ptr(stream)))
     return ids, src, scores
 
+
+
+_PLAN_FIELDS = ("grid", "block_n", "cluster", "dual", "qt", "uqt", "nt", "win", "pmax",
+                "stages", "smem", "scratch", "sets")
+
+
+def plan_search(n: int, d: int, q: int, k: int, num_sms: int = 148, force_block_n: int = 0,
+                force_pair: int = 0, pair_capacity: int = 74) -> dict:
+    """Host-side plan of a tensor-core search (no device work, no GPU needed):
+    launch shape, schedule, shared memory and list scratch."""
+    out = (ctypes.c_int64 * len(_PLAN_FIELDS))()
+    check(_lib.load().oprag_plan_search(n, d, q, k, num_sms, force_block_n, force_pair,
+                                        pair_capacity, out))
+    return dict(zip(_PLAN_FIELDS, (int(v) for v in out)))
