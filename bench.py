@@ -101,6 +101,23 @@ def workload_name(cfg: int, w, dense_first: int = 0) -> str:
     return f"{base}: {w.n} x {w.d} {w.dtype}, {w.q} queries/step"
 
 
+def slowest_replica(totals_ms, world: int, device):
+    """Each timed total maximised over the ranks: the replicas run the same
+    steps side by side, so the slowest one sets the job's time (identity for
+    one rank).  Collective over the default process group."""
+    if world <= 1:
+        return [float(t) for t in totals_ms]
+    import torch
+    t = torch.tensor([float(x) for x in totals_ms], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return [float(x) for x in t]
+
+
+def job_rate(q: int, steps: int, world: int, total_ms: float) -> float:
+    """Whole-job queries/s: every rank searched q queries per step."""
+    return q * steps * world / (total_ms * 1e-3)
+
+
 def roofline_terms(w, cfg, dense_first: int = 0):
     """Algorithmic bytes and flops of one search-kernel launch."""
     elem = 4 if w.dtype == "f32" else 2
@@ -452,12 +469,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
             if i >= args.warmup:
                 e2e_ms.append((time.perf_counter() - t0) * 1e3)
 
-    total_ms = sum(step_ms)
-    e2e_total = sum(e2e_ms)
-    if world > 1:
-        tt = torch.tensor([total_ms, e2e_total], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        total_ms, e2e_total = float(tt[0]), float(tt[1])
+    total_ms, e2e_total = slowest_replica([sum(step_ms), sum(e2e_ms)], world, dev)
     if rank != 0:
         return None
 
@@ -497,7 +509,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
     roof["traffic"] = ncu_traffic(key)
 
     queries_all = w.q * args.steps * world
-    value = queries_all / (total_ms * 1e-3)
+    value = job_rate(w.q, args.steps, world, total_ms)
     h2d = w.q * w.d * (2 if elem_bf16 else 4)
     if cfg == 4:
         h2d += 4096 * (w.d * 2 + 8)
