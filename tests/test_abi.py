@@ -71,6 +71,13 @@ def test_null_and_shape_arguments_are_rejected_on_the_host(lib):
     assert lib.oprag_index_check(None) == -1
     assert lib.oprag_index_info(None, None, None, None, None) == -1
     assert lib.oprag_index_last_path(None) == 0
+    t = ctypes.c_int32()
+    assert lib.oprag_index_last_tiles_per_cta(None, ctypes.byref(t)) == -1
+    assert lib.oprag_index_last_launch(None, None, None, None) == -1
+    plan = (ctypes.c_int64 * 13)()
+    assert lib.oprag_plan_search(1000, 768, 16, 5, 148, 0, 0, 74, None) == -1
+    assert lib.oprag_plan_search(1000, 768, 16, 5, 0, 0, 0, 74, plan) == -1
+    assert lib.oprag_plan_search(1000, 768, 16, 5, 148, 0, 0, 74, plan) == 0
     lib.oprag_index_destroy(None)
 
 
