@@ -2,11 +2,15 @@
 """Throughput of the GB300 retrieval hot path: queries/s at top-k and the
 fraction of the roofline reached by the dominant kernel.
 
-Default workload (one step = one search call): the paper-shaped dense top-5
-search, 32768 chunks x 768 bf16, a batch of 256 queries (Sec. 5.1 shapes:
-32K chunks, 768-d embeddings).  --config/--batch select the other workloads
-(0 tiny fp32, 2 clustered 4096 queries, 3 hybrid 1024 queries, 4 scale 1M
-chunks with a 4096-row upsert before each 2048-query search).
+Headline workload (one step = one 4096-row upsert + one search call): the
+scale case, 1,048,576 chunks x 768 bf16, a batch of 2048 queries, top-100
+(the largest single-GPU workload; Sec. 5.1 shapes: 768-d embeddings, dense
+retrieval with upserts between batches).  The same JSON line carries, under
+"configs", the other workloads measured the same way: the tiny fp32 case
+(1024 x 384, 16 queries), the paper-shaped dense search (32768 x 768, batches
+of 1, 32 and 256, top-5), the clustered search (32768 x 1024, 4096 queries,
+top-10) and the hybrid dense + BM25 search (32768 x 768, 1024 queries, top-5).
+--config C [--batch Q] measures one workload alone.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
@@ -14,10 +18,16 @@ Timing: W untimed steps, then K steps; before every step a 512 MiB buffer is
 written (L2 flush, outside the timed events); each step is bracketed by CUDA
 events on the launch stream and the steps are enqueued without waiting on the
 host.  A second pass over the same steps, with the library's own events
-around each of its kernels, times the search kernel for the roofline.  Under torchrun every rank runs the same workload on
-its own GPU (replicas), the slowest rank's time counts and `value` adds the
-queries of all ranks.  --impl reference times the CPU oracle on the host cores
-(bounded samples of the same workload).
+around each of its kernels, times the search kernel for the roofline.  Under
+torchrun every rank runs the same workloads on its own GPU (replicas), the
+slowest rank's time counts and `value` adds the queries of all ranks.
+
+Oracle leg (skipped with --no-cpu-baseline): on rank 0 the outputs of the
+last timed step of every workload are checked against the CPU oracle on a
+sample with rows in every 32-query group of every 128-query tile
+("parity"), and the oracle itself is timed on a bounded sample of the
+headline workload ("cpu_baseline").  --impl reference times the oracle alone
+on the host cores (bounded samples of the same workload).
 """
 from __future__ import annotations
 
@@ -60,15 +70,24 @@ def source_hash(read=None) -> str:
     return h.hexdigest()[:16]
 
 
-def parse():
+HEADLINE = (4, 2048)
+# The other workloads reported under "configs": (config, queries per step).
+SUB_WORKLOADS = [(0, 16), (1, 1), (1, 32), (1, 256), (2, 4096), (3, 1024)]
+TOL = 1e-4          # parity bar: absolute score tolerance (oracle/check.py rules)
+
+
+def parse(argv=None):
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=200)
-    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--steps", type=int, default=50)
+    p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    p.add_argument("--config", type=int, default=1)
-    p.add_argument("--batch", type=int, default=None)
-    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--config", type=int, default=None,
+                   help="measure this workload alone (default: the scale workload as the "
+                        "headline plus every other workload under \"configs\")")
+    p.add_argument("--batch", type=int, default=None, help="queries per step (with --config)")
+    p.add_argument("--no-cpu-baseline", action="store_true",
+                   help="skip the oracle leg (parity of the timed outputs and cpu_baseline)")
     p.add_argument("--block-n", type=int, default=0, help="tensor-core tile rows (0 = auto)")
     p.add_argument("--path", choices=["auto", "simt", "tc"], default="auto")
     p.add_argument("--pair", choices=["auto", "single", "pair", "dual"], default="auto",
@@ -86,7 +105,7 @@ def parse():
     p.add_argument("--dense-first", type=int, default=0, metavar="N",
                    help="config 3 only: dense top-N, then the lexical rerank of those N "
                         "candidates (dense-first hybrid) instead of the full hybrid")
-    return p.parse_args()
+    return p.parse_args(argv)
 
 
 def default_batch(cfg: int) -> int:
@@ -99,6 +118,36 @@ def workload_name(cfg: int, w, dense_first: int = 0) -> str:
     if cfg == 3 and dense_first:
         base = f"dense-first hybrid top-5 (dense top-{dense_first}, lexical rerank)"
     return f"{base}: {w.n} x {w.d} {w.dtype}, {w.q} queries/step"
+
+
+def workload_key(cfg: int, q: int) -> str:
+    return f"cfg{cfg}_q{q}"
+
+
+def config_dict(cfg: int, w, world: int, dense_first: int = 0) -> dict:
+    """The `config` object of a bench line; the same for both arms."""
+    return {"workload": workload_name(cfg, w, dense_first), "config_index": cfg,
+            "n": w.n, "d": w.d, "q": w.q, "k": w.k, "parallelism": f"replicas{world}",
+            "l2": f"flushed before every step ({L2_FLUSH_BYTES >> 20} MiB write)"}
+
+
+def parity_rows(q: int, seed: int = 0) -> np.ndarray:
+    """Rows to check against the oracle: every row of a batch of at most 64
+    queries; otherwise one random row in every 32-query group of every
+    128-query tile (each TMEM lane quarter of each tile)."""
+    if q <= 64:
+        return np.arange(q)
+    rng = np.random.default_rng(seed)
+    rows = []
+    for lo in range(0, q, 32):
+        rows.append(int(rng.integers(lo, min(q, lo + 32))))
+    return np.asarray(rows, np.int64)
+
+
+def upsert_sequence(warmup: int, steps: int, rounds: int = 4):
+    """Upsert rounds applied before the last timed step's search, in order
+    (step i upserts round i mod rounds; warm-up steps first)."""
+    return [i % rounds for i in range(warmup)] + [i % rounds for i in range(steps)]
 
 
 def slowest_replica(totals_ms, world: int, device):
@@ -118,14 +167,28 @@ def job_rate(q: int, steps: int, world: int, total_ms: float) -> float:
     return q * steps * world / (total_ms * 1e-3)
 
 
+def sparse_terms(w) -> dict:
+    """Postings (chunk, weight) pairs the lexical half must read: those of the
+    distinct query terms (each read at least once), and the total visited
+    over all queries (a term repeated in a query counts again)."""
+    doc = np.repeat(np.arange(w.n, dtype=np.int64), np.diff(w.doc_indptr.astype(np.int64)))
+    pairs = np.unique(doc * w.vocab + w.doc_terms.astype(np.int64))
+    df = np.bincount(pairs % w.vocab, minlength=w.vocab)
+    distinct = np.unique(w.q_terms)
+    return {"postings_distinct_terms": int(df[distinct].sum()),
+            "postings_visited": int(df[w.q_terms].sum()),
+            "bytes_distinct_terms": int(df[distinct].sum()) * 8,
+            "posting_bytes": 8}
+
+
 def roofline_terms(w, cfg, dense_first: int = 0):
-    """Algorithmic bytes and flops of one search-kernel launch."""
+    """Algorithmic bytes and flops of one search call: the corpus and the
+    queries read once (plus, for the hybrid search, the postings of the
+    distinct query terms), and 2 q n d multiply-adds of the dense scores."""
     elem = 4 if w.dtype == "f32" else 2
-    corpus = w.n * w.d * elem
-    queries = w.q * w.d * elem
-    nbytes = corpus + queries
+    nbytes = w.n * w.d * elem + w.q * w.d * elem
     if cfg == 3 and not dense_first:
-        nbytes += w.q * ((w.n + 3) // 4 * 4) * 4      # fused epilogue reads the BM25 block
+        nbytes += sparse_terms(w)["bytes_distinct_terms"]
     flops = 2.0 * w.q * w.n * w.d
     return nbytes, flops
 
@@ -284,38 +347,34 @@ class NvmlSampler:
                 "samples": len(self.samples), "source": "nvml, 2 ms, timed region"}
 
 
-def make_inputs(cfg: int, batch: int):
-    if cfg == 4:
-        w = workloads.config(4, batch=batch)
-    else:
-        w = workloads.config(cfg, batch=batch)
-    return w
-
-
 # --------------------------------------------------------------------- ours
 
-def run_ours(args, rank: int, world: int, local_rank: int):
+def _to_dev(a, dev):
+    import torch
+    if a.dtype == np.uint16:
+        return torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).to(dev)
+    return torch.from_numpy(a).to(dev)
+
+
+def _to_pinned(a):
+    import torch
+    t = (torch.from_numpy(a.view(np.int16)).view(torch.bfloat16) if a.dtype == np.uint16
+         else torch.from_numpy(a))
+    return t.pin_memory()
+
+
+def measure(args, cfg: int, batch: int, rank: int, world: int, local_rank: int,
+            dense_first: int = 0):
+    """Times one workload on this rank's GPU.  Returns (result, w, extra) on
+    rank 0 (None elsewhere); extra holds the last timed step's outputs and
+    what the oracle leg needs to rebuild the index it searched."""
     import torch
     from paper_2608_08340_gb300.index import Index
 
-    torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-    cfg = args.config
-    dense_first = args.dense_first if cfg == 3 else 0
-    batch = args.batch or default_batch(cfg)
-    w = make_inputs(cfg, batch)
-
-    def to_dev(a):
-        if a.dtype == np.uint16:
-            return torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).to(dev)
-        return torch.from_numpy(a).to(dev)
-
-    def to_pinned(a):
-        t = (torch.from_numpy(a.view(np.int16)).view(torch.bfloat16) if a.dtype == np.uint16
-             else torch.from_numpy(a))
-        return t.pin_memory()
-
-    idx = Index(to_dev(w.E_data))
+    dense_first = dense_first if cfg == 3 else 0
+    w = workloads.config(cfg, batch=batch)
+    idx = Index(_to_dev(w.E_data, dev))
     if cfg == 3:
         idx.set_sparse(w.doc_indptr, w.doc_terms, w.vocab, w.k1, w.b)
         q_indptr = torch.from_numpy(w.q_indptr).to(dev)
@@ -325,15 +384,16 @@ def run_ours(args, rank: int, world: int, local_rank: int):
     idx.force_pair(None if args.pair == "auto" else args.pair)
     idx.reserve(w.q, w.k)
     use_graph = args.graph and cfg in (0, 1, 2)
+    prev_stream = torch.cuda.current_stream()
     if use_graph:
         from paper_2608_08340_gb300 import _lib
         idx.set_option(_lib.OPRAG_OPT_GRAPH, 1)
         side = torch.cuda.Stream()
-        side.wait_stream(torch.cuda.current_stream())
+        side.wait_stream(prev_stream)
         torch.cuda.set_stream(side)              # every launch of the run goes to it
     idx.enable_timing(True)
-    Q = to_dev(w.Q_data)
-    Qh = to_pinned(w.Q_data)
+    Q = _to_dev(w.Q_data, dev)
+    Qh = _to_pinned(w.Q_data)
     ids = torch.empty((w.q, w.k), dtype=torch.int64, device=dev)
     scores = torch.empty((w.q, w.k), dtype=torch.float32, device=dev)
     ids_h = torch.empty((w.q, w.k), dtype=torch.int64).pin_memory()
@@ -342,36 +402,37 @@ def run_ours(args, rank: int, world: int, local_rank: int):
     if cfg == 4:
         for r in range(4):
             u_ids, u_rows = workloads.upsert_batch(w.n, w.d, 4096, r + 1, w.dtype)
-            ups.append((u_ids, to_dev(u_rows), to_pinned(u_rows)))
+            ups.append((u_ids, u_rows, _to_dev(u_rows, dev), _to_pinned(u_rows)))
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
     stream = torch.cuda.current_stream()      # the side stream in graph mode
+    last = {}
 
     def step(i, host=False):
         if cfg == 4:
-            u_ids, u_dev, u_host = ups[i % len(ups)]
+            u_ids, _, u_dev, u_host = ups[i % len(ups)]
             idx.upsert(u_ids, u_host if host else u_dev)
         if host:
-            if cfg == 3:
-                raise RuntimeError("unreachable")
             idx.search_host(Qh, w.k, out=(ids_h, scores_h))
         elif cfg == 3 and dense_first:
-            idx.hybrid_search_dense_first(Q, q_indptr, q_terms, w.alpha, dense_first, w.k)
+            last["out"] = idx.hybrid_search_dense_first(Q, q_indptr, q_terms, w.alpha,
+                                                        dense_first, w.k)
         elif cfg == 3:
-            idx.hybrid_search(Q, q_indptr, q_terms, w.alpha, w.k)
+            last["out"] = idx.hybrid_search(Q, q_indptr, q_terms, w.alpha, w.k)
         else:
             idx.search(Q, w.k, out=(ids, scores))
+            last["out"] = (ids, scores)
 
-    # search + merge; k > 32 adds the sampled first pass (search + merge);
-    # config 3 adds the BM25 pass (dense-first: the dense top-N search, with
-    # the sampled pass for N > 32, and the rerank), config 4 the upsert scatter.
-    k_search = dense_first if dense_first else w.k
-    launches_per_step = 2 + (2 if k_search > 32 else 0) + (1 if cfg in (3, 4) else 0)
-
+    # our kernels per step: search + merge; k > 32 over many tiles adds the
+    # sampled first pass (search + merge); config 3 adds the BM25 pass
+    # (dense-first: the rerank), config 4 the upsert scatter.
     for i in range(args.warmup):
         flush.zero_()
         step(i)
     torch.cuda.synchronize()
     idx.check()
+    t = idx.last_timing()
+    sampled = t["sample_ms"] > 0.0
+    launches_per_step = 2 + (2 if sampled else 0) + (1 if cfg in (3, 4) else 0)
 
     if world > 1:
         torch.distributed.barrier()
@@ -395,19 +456,20 @@ def run_ours(args, rank: int, world: int, local_rank: int):
     if world > 1:
         torch.distributed.barrier()
     idx.check()
+    # The last timed step's outputs, kept for the oracle leg.
+    out_ids, out_scores = (x.cpu().numpy() for x in last["out"])
 
     # Per-kernel breakdown (roofline): the same steps again with events around
-    # each kernel of the search; these events also separate the search and
-    # merge launches, so they are not used for the step time.
+    # each kernel of the search; these events also separate the launches, so
+    # they are not used for the step time.
     idx.enable_timing(True)
-    search_ms, lex_ms, merge_ms = [], [], []
+    tim = {"search_ms": [], "merge_ms": [], "lexical_ms": [], "sample_ms": []}
     for i in range(min(args.steps, 50)):
         flush.zero_()
         step(i)
         t = idx.last_timing()              # waits for this step
-        search_ms.append(t["search_ms"])
-        merge_ms.append(t["merge_ms"])
-        lex_ms.append(t["lexical_ms"])
+        for key in tim:
+            tim[key].append(t[key])
     idx.enable_timing(False)
     idx.check()
 
@@ -427,11 +489,11 @@ def run_ours(args, rank: int, world: int, local_rank: int):
     upsert_ms = []
     if cfg == 4:
         for i in range(min(args.steps, 20)):
-            u_ids, u_dev, _ = ups[i % len(ups)]
+            _, _, u_dev, _ = ups[i % len(ups)]
             a = torch.cuda.Event(enable_timing=True)
             b = torch.cuda.Event(enable_timing=True)
             a.record(stream)
-            idx.upsert(u_ids, u_dev)
+            idx.upsert(ups[i % len(ups)][0], u_dev)
             b.record(stream)
             upsert_ms.append((a, b))
         torch.cuda.synchronize()
@@ -470,6 +532,24 @@ def run_ours(args, rank: int, world: int, local_rank: int):
                 e2e_ms.append((time.perf_counter() - t0) * 1e3)
 
     total_ms, e2e_total = slowest_replica([sum(step_ms), sum(e2e_ms)], world, dev)
+    quality = None
+    if dense_first and rank == 0:
+        # Quality against the full hybrid search (Sec. 5.2 Recall@k; Jaccard
+        # overlap of the two top-k sets), as the paper reports for this policy.
+        f_ids, _ = idx.hybrid_search(Q, q_indptr, q_terms, w.alpha, w.k)
+        d_ids, _ = idx.hybrid_search_dense_first(Q, q_indptr, q_terms, w.alpha, dense_first, w.k)
+        f_ids, d_ids = f_ids.cpu().numpy(), d_ids.cpu().numpy()
+        inter = [len(set(a) & set(b)) for a, b in zip(f_ids.tolist(), d_ids.tolist())]
+        union = [len(set(a) | set(b)) for a, b in zip(f_ids.tolist(), d_ids.tolist())]
+        quality = {"recall_at_k": float(np.mean(inter)) / w.k,
+                   "jaccard": float(np.mean([i / u for i, u in zip(inter, union)])),
+                   "vs": "full hybrid search on the same batch", "n_candidates": dense_first}
+    path, launch = idx.last_path, idx.last_launch
+    idx.close()
+    if use_graph:
+        torch.cuda.set_stream(prev_stream)
+    del flush
+    torch.cuda.empty_cache()
     if rank != 0:
         return None
 
@@ -478,13 +558,13 @@ def run_ours(args, rank: int, world: int, local_rank: int):
     # The burst figure is for a kernel timed alone; when the timed loop kept
     # the GPU at its power cap (NVML reported sw_power_cap while it ran), the
     # sustained figure (the same GEMM back to back under the cap) applies.
-    capped = "sw_power_cap" in clocks.summary().get("reasons", [])
+    clk = clocks.summary()
+    capped = "sw_power_cap" in clk.get("reasons", [])
     tflops = tflops_sustained if capped else tflops_burst
-    t_kernel = statistics.mean(search_ms) * 1e-3
+    t_kernel = statistics.mean(tim["search_ms"]) * 1e-3
     t_bytes = nbytes / (hbm * 1e9)
     t_flops = flops / (tflops * 1e12)
-    elem_bf16 = w.dtype == "bf16"
-    if t_flops > t_bytes and elem_bf16:
+    if t_flops > t_bytes and w.dtype == "bf16":
         roof = {"bound": "tensor", "achieved": flops / t_kernel / 1e12, "peak": tflops,
                 "unit": "TFLOP/s"}
     else:
@@ -494,37 +574,37 @@ def run_ours(args, rank: int, world: int, local_rank: int):
     if roof["bound"] == "tensor":
         roof["peak_kind"] = ("sustained: sw_power_cap active in the timed region" if capped
                              else "burst")
-    roof["kernel"] = "tc_search_kernel" if idx.last_path == "tc" else "simt_search_kernel"
-    roof["kernel_ms_mean"] = statistics.mean(search_ms)
-    roof["kernel_ms_median"] = statistics.median(search_ms)
-    roof["merge_ms_mean"] = statistics.mean(merge_ms)
-    roof["merge_ms_median"] = statistics.median(merge_ms)
-    if cfg == 3:
-        roof["bm25_ms_mean"] = statistics.mean(lex_ms)
-        roof["bm25_ms_median"] = statistics.median(lex_ms)
+    roof["kernel"] = "tc_search_kernel" if path == "tc" else "simt_search_kernel"
+    roof["kernel_ms_mean"] = statistics.mean(tim["search_ms"])
+    roof["kernel_ms_median"] = statistics.median(tim["search_ms"])
+    roof["merge_ms_mean"] = statistics.mean(tim["merge_ms"])
+    if sampled:
+        # k > 32: the first pass over every 16th corpus tile and its merge,
+        # timed apart from the main pass (the dominant kernel above)
+        roof["sample_pass_ms_mean"] = statistics.mean(tim["sample_ms"])
+    if cfg == 3 and not dense_first:
+        roof["bm25_ms_mean"] = statistics.mean(tim["lexical_ms"])
+        roof["sparse"] = sparse_terms(w)
     roof["algorithmic_bytes"] = nbytes
     roof["algorithmic_flops"] = flops
-    roof["roofline_time_frac"] = max(t_bytes, t_flops) / (statistics.mean(step_ms) * 1e-3)
-    key = f"cfg{cfg}_q{w.q}"
-    roof["traffic"] = ncu_traffic(key)
+    # the whole step against the roofline of its algorithmic work
+    roof["step_frac"] = max(t_bytes, t_flops) / (statistics.mean(step_ms) * 1e-3)
+    roof["traffic"] = ncu_traffic(workload_key(cfg, w.q))
 
     queries_all = w.q * args.steps * world
-    value = job_rate(w.q, args.steps, world, total_ms)
-    h2d = w.q * w.d * (2 if elem_bf16 else 4)
+    h2d = w.q * w.d * (2 if w.dtype == "bf16" else 4)
     if cfg == 4:
         h2d += 4096 * (w.d * 2 + 8)
     if cfg == 3:
         h2d += w.q_indptr.nbytes + w.q_terms.nbytes
     d2h = w.q * w.k * 12
     result = {
-        "metric": f"queries/s at top-{w.k}", "value": value, "unit": "queries/s",
-        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "metric": f"queries/s at top-{w.k}", "value": job_rate(w.q, args.steps, world, total_ms),
+        "unit": "queries/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": total_ms / args.steps,
         "ms_per_step_median": statistics.median(step_ms), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": w.dtype, "data": "synthetic",
-        "config": {"workload": workload_name(cfg, w, dense_first), "config_index": cfg,
-                   "n": w.n, "d": w.d, "q": w.q, "k": w.k, "parallelism": f"replicas{world}",
-                   "l2": f"flushed before every step ({L2_FLUSH_BYTES >> 20} MiB write)"},
+        "config": config_dict(cfg, w, world, dense_first),
         "roofline": roof,
         "e2e": {"value": queries_all / (e2e_total * 1e-3), "unit": "queries/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
@@ -535,33 +615,76 @@ def run_ours(args, rank: int, world: int, local_rank: int):
                     "ms_per_step_median": statistics.median(warm_ms), "steps": len(warm_ms),
                     "l2": "not flushed between steps"},
         "gpu_launches": launches_per_step * args.steps,
-        "clocks": dict(clocks.summary(), smi=smi.summary()),
-        "path": idx.last_path,
-        "launch": idx.last_launch,
-        "graph_mode": bool(use_graph),
+        "clocks": dict(clk, smi=smi.summary()),
+        "path": path, "launch": launch, "graph_mode": bool(use_graph),
     }
     if upsert_ms:
         # Sec. 3.2 Op_upsert: 4096 rows of d bf16 plus their int64 ids per call.
         ub = 4096 * (w.d * 2 + 8)
         result["upsert"] = {"rows": 4096, "bytes": ub, "ms_median": statistics.median(upsert_ms),
                             "GB_per_s": ub / (statistics.median(upsert_ms) * 1e-3) / 1e9}
-    if dense_first:
-        # Quality against the full hybrid search (Sec. 5.2 Recall@k; Jaccard
-        # overlap of the two top-k sets), as the paper reports for this policy.
-        f_ids, _ = idx.hybrid_search(Q, q_indptr, q_terms, w.alpha, w.k)
-        d_ids, _ = idx.hybrid_search_dense_first(Q, q_indptr, q_terms, w.alpha, dense_first, w.k)
-        f_ids, d_ids = f_ids.cpu().numpy(), d_ids.cpu().numpy()
-        inter = [len(set(a) & set(b)) for a, b in zip(f_ids.tolist(), d_ids.tolist())]
-        union = [len(set(a) | set(b)) for a, b in zip(f_ids.tolist(), d_ids.tolist())]
-        result["quality"] = {"recall_at_k": float(np.mean(inter)) / w.k,
-                             "jaccard": float(np.mean([i / u for i, u in zip(inter, union)])),
-                             "vs": "full hybrid search on the same batch",
-                             "n_candidates": dense_first}
-    idx.close()
-    return result, w
+    if quality:
+        result["quality"] = quality
+    extra = {"ids": out_ids, "scores": out_scores,
+             "upserts": ([(ups[r][0], ups[r][1]) for r in upsert_sequence(args.warmup, args.steps)]
+                         if cfg == 4 else [])}
+    return result, w, extra
 
 
-# --------------------------------------------------------------------- oracle
+def sub_entry(res: dict) -> dict:
+    """The fields of a workload's line kept under the headline's "configs"."""
+    keep = ("value", "unit", "ms_per_step", "ms_per_step_median", "roofline", "e2e", "clocks",
+            "warm_l2", "parity", "gpu_launches", "path", "launch", "upsert", "metric")
+    out = {k: res[k] for k in keep if k in res}
+    out["workload"] = res["config"]["workload"]
+    return out
+
+
+# --------------------------------------------------------------------- oracle leg
+
+def parity_check(w, cfg: int, extra: dict, threads: int) -> dict:
+    """The last timed step's outputs against the CPU oracle (oracle/check.py
+    rules: scores within 1e-4, ids exact outside near-tie blocks) on the rows
+    of parity_rows(); for the scale workload the oracle searches the index as
+    the timed upserts left it."""
+    import oracle
+    from oracle import check
+
+    rows = parity_rows(w.q, seed=cfg)
+    E = w.E_data
+    if extra["upserts"]:
+        E = E.copy()
+        for u_ids, u_rows in extra["upserts"]:
+            oracle.upsert(E, u_ids, u_rows)
+    Qs = w.Q_data[rows]
+    if cfg == 3:
+        qts = [w.q_terms[w.q_indptr[r]:w.q_indptr[r + 1]] for r in rows]
+        qip = np.zeros(len(rows) + 1, np.int32)
+        qip[1:] = np.cumsum([len(t) for t in qts])
+        qtm = np.concatenate(qts).astype(np.int32)
+
+        def fn(kout):
+            return oracle.hybrid_search(E, Qs, w.doc_indptr, w.doc_terms, w.vocab, qip, qtm,
+                                        w.alpha, kout, w.k1, w.b, nthreads=threads)
+    else:
+        def fn(kout):
+            return oracle.search(E, Qs, kout, nthreads=threads)
+    t0 = time.perf_counter()
+    out = {"rows_checked": int(len(rows)), "of": int(w.q),
+           "sample": ("every query" if len(rows) == w.q else
+                      "one random query in every 32-query group of every 128-query tile"),
+           "tol": TOL}
+    try:
+        o_ids, o_sc = check.topk_with_margin(fn, w.k, w.n, TOL)
+        stats = check.check_topk(extra["ids"][rows], extra["scores"][rows], o_ids, o_sc, w.k,
+                                 TOL, n=w.n, query_index=rows, label=workload_key(cfg, w.q))
+        out.update(passed=True, exact_id_lists=stats["exact_id_lists"],
+                   max_abs_score_err=stats["max_abs_score_err"])
+    except check.TopkMismatch as e:
+        out.update(passed=False, error=str(e)[:400])
+    out["oracle_s"] = round(time.perf_counter() - t0, 2)
+    return out
+
 
 def oracle_queries_per_s(w, cfg, nq: int, threads: int, offset: int = 0):
     import oracle
@@ -584,7 +707,7 @@ def cpu_baseline(w, cfg, budget_s: float = 12.0):
     """The oracle as it stands, on all host cores, on a bounded sample sized
     from a short pilot to about budget_s seconds."""
     threads = os.cpu_count() or 1
-    pilot = max(threads, 8)
+    pilot = threads
     rate = oracle_queries_per_s(w, cfg, pilot, threads)
     nq = int(min(max(pilot, rate * budget_s), 4 * w.q))
     nq = max(threads, nq // threads * threads)
@@ -595,19 +718,35 @@ def cpu_baseline(w, cfg, budget_s: float = 12.0):
 
 
 def run_reference(args):
-    cfg = args.config
-    batch = args.batch or default_batch(cfg)
-    w = make_inputs(cfg, batch)
+    """The reference arm: the oracle (the CPU definition of the path) on the
+    host cores, on bounded samples of the same workload and config as ours.
+    The scale workload's step applies its 4096-row upsert to the oracle's
+    array before searching, as ours does."""
+    import oracle
+    cfg = HEADLINE[0] if args.config is None else args.config
+    batch = args.batch or (HEADLINE[1] if args.config is None else default_batch(cfg))
+    w = workloads.config(cfg, batch=batch)
     threads = os.cpu_count() or 1
+    E = w.E_data.copy() if cfg == 4 else w.E_data
+    ups = [workloads.upsert_batch(w.n, w.d, 4096, r + 1, w.dtype) for r in range(4)] if cfg == 4 else []
+    ww = workloads.Workload(w.name, w.dtype, w.k, E, w.Q_data, w.doc_indptr, w.doc_terms,
+                            w.q_indptr, w.q_terms, w.vocab, w.k1, w.b, w.alpha)
     # each step: a bounded sample of the step's queries (whole run within minutes)
-    pilot = oracle_queries_per_s(w, cfg, max(threads, 8), threads)
-    per_step = int(max(threads, min(w.q, pilot * 4.0)))
-    times, done = [], 0
+    pilot = oracle_queries_per_s(ww, cfg, threads, threads)
+    per_step = int(max(threads, min(w.q, pilot * 2.0)) // threads * threads)
+
+    def one(i, nq):
+        if ups:
+            u_ids, u_rows = ups[i % len(ups)]
+            oracle.upsert(E, u_ids, u_rows)
+        oracle_queries_per_s(ww, cfg, nq, threads, offset=i * nq)
+
     for i in range(args.warmup):
-        oracle_queries_per_s(w, cfg, threads, threads)
+        one(i, threads)
+    times, done = [], 0
     for i in range(args.steps):
         t0 = time.perf_counter()
-        oracle_queries_per_s(w, cfg, per_step, threads, offset=i * per_step)
+        one(i, per_step)
         times.append(time.perf_counter() - t0)
         done += per_step
     value = done / sum(times)
@@ -616,11 +755,11 @@ def run_reference(args):
         "unit": "queries/s", "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1e3 * sum(times) / len(times), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": workload_name(cfg, w), "config_index": cfg, "n": w.n, "d": w.d,
-                   "q": w.q, "k": w.k, "parallelism": "host threads"},
+        "config": config_dict(cfg, w, args.gpus),
         "cpu_baseline": {"value": value, "unit": "queries/s", "cores": threads,
                          "kind": "oracle",
-                         "sample": f"{per_step} queries per step of the {w.q}-query batch"},
+                         "sample": f"{per_step} queries per step of the {w.q}-query batch"
+                                   + (", after the step's 4096-row upsert" if ups else "")},
         "e2e": {"value": value, "unit": "queries/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -755,20 +894,40 @@ def main():
         if rank == 0:
             run_reference(args)
         return
+    import torch
+    torch.cuda.set_device(local_rank)
     if world > 1:
-        import torch
-        torch.cuda.set_device(local_rank)
         torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
-    res = run_ours(args, rank, world, local_rank)
+    oracle_leg = not args.no_cpu_baseline and rank == 0
+    threads = os.cpu_count() or 1
+    if args.config is None:
+        plan = [HEADLINE] + SUB_WORKLOADS
+    else:
+        plan = [(args.config, args.batch or default_batch(args.config))]
+    head = None
+    subs = {}
+    for n_run, (cfg, batch) in enumerate(plan):
+        res = measure(args, cfg, batch, rank, world, local_rank,
+                      dense_first=args.dense_first if n_run == 0 else 0)
+        if res is None:
+            continue
+        result, w, extra = res
+        if oracle_leg:
+            result["parity"] = parity_check(w, cfg, extra, threads)
+            if n_run == 0:
+                result["cpu_baseline"] = cpu_baseline(w, cfg)
+        if n_run == 0:
+            head = result
+        else:
+            subs[workload_key(cfg, batch)] = sub_entry(result)
+        del w, extra
     if world > 1:
-        import torch
         torch.distributed.destroy_process_group()
-    if res is None:
+    if head is None:
         return
-    result, w = res
-    if not args.no_cpu_baseline:
-        result["cpu_baseline"] = cpu_baseline(w, args.config)
-    print(json.dumps(result))
+    if subs:
+        head["configs"] = subs
+    print(json.dumps(head))
 
 
 if __name__ == "__main__":

@@ -93,9 +93,13 @@ OPRAG_API const void *oprag_index_data(const oprag_index *idx);
 OPRAG_API int oprag_index_get_rows(const oprag_index *idx, int64_t first, int64_t count, void *out);
 
 /*
- * Pre-allocates the scratch memory that searches of up to q_max queries and
- * k_max results need, so that later calls allocate nothing.  Optional: search
- * calls grow the scratch on demand (which synchronises the device once).
+ * Pre-allocates the scratch memory that dense searches of up to q_max queries
+ * and k_max results need -- partial lists, the sampled first pass of k > 32,
+ * the per-query shared bounds (zeroed here) and, with a sparse side, the
+ * lexical block of the hybrid search -- so that later searches of that size
+ * allocate nothing and never synchronise the device.  Optional: search calls
+ * grow the scratch on demand (which synchronises the device once).
+ * Synchronous.
  */
 OPRAG_API int oprag_index_reserve(oprag_index *idx, int32_t q_max, int32_t k_max);
 
@@ -275,19 +279,38 @@ OPRAG_API int oprag_index_set_option(oprag_index *idx, int32_t option, int32_t v
 #define OPRAG_OPT_GRAPH 6
 
 /* OPRAG_OPT_TIMING: 1 makes every later search record CUDA events, on the
- * call's stream, around its lexical (BM25) kernel, its main search kernel and
- * its merge kernel; oprag_index_last_timing() reads them.  0 (default) off. */
+ * call's stream, around its lexical (BM25) kernel, its sampled first pass,
+ * its main search kernel and its merge kernel; oprag_index_last_timing()
+ * reads them.  0 (default) off. */
 #define OPRAG_OPT_TIMING 3
+
+/* OPRAG_OPT_WAIT_LIMIT (test hook): the number of clock cycles a wait of the
+ * tensor-core search kernel on one of its pipeline barriers may spin before
+ * the kernel gives up, records OPRAG_ERR_DEVICE for oprag_index_check,
+ * drains its copies and tensor-core work, frees its tensor memory and
+ * returns (the results of that search are then undefined).  0 (default)
+ * means about 2^31 cycles (about a second); a small value lets a test make
+ * the waits of a real search run out. */
+#define OPRAG_OPT_WAIT_LIMIT 7
 
 /*
  * Device durations (milliseconds) of the kernels of the last search issued
  * with timing on: lexical_ms (BM25 pass of a hybrid search, 0 for a dense
- * search), search_ms (score contraction + fused selection), merge_ms (final
- * top-k reduction).  Waits for that search to finish.  Any out-pointer may be
- * NULL.  OPRAG_ERR_NOT_READY if no timed search was issued.
+ * search), sample_ms (the first pass over every 16th corpus tile and its
+ * merge that a search with k > 32 over a large corpus runs first, else 0),
+ * search_ms (main pass: score contraction + fused selection), merge_ms
+ * (final top-k reduction).  Waits for that search to finish.  Any
+ * out-pointer may be NULL.  OPRAG_ERR_NOT_READY if no timed search was issued.
  */
-OPRAG_API int oprag_index_last_timing(oprag_index *idx, float *lexical_ms, float *search_ms,
-                                      float *merge_ms);
+OPRAG_API int oprag_index_last_timing(oprag_index *idx, float *lexical_ms, float *sample_ms,
+                                      float *search_ms, float *merge_ms);
+
+/* Bytes currently held by the index's grow-on-demand buffers: the search
+ * scratch (partial lists, sampled pass), the shared per-query k-th bounds
+ * and the lexical block of the hybrid search.  Any out-pointer may be NULL.
+ * For tests of oprag_index_reserve. */
+OPRAG_API int oprag_index_buffer_bytes(const oprag_index *idx, int64_t *scratch, int64_t *bounds,
+                                       int64_t *lexical);
 
 /* Which kernel family served the last search on this index: 1 SIMT, 2 tensor
  * core, 0 none yet. */
@@ -328,21 +351,26 @@ OPRAG_API int oprag_plan_search(int64_t n, int32_t d, int32_t q, int32_t k, int3
  * claimed the GPU, or a host that cannot afford the device-wide
  * synchronisation that cudaMalloc / cudaFree may cause.
  *
- * Same arguments, results and stream semantics as oprag_search.  Instead of
- * the index's scratch buffer (which oprag_search grows with cudaMalloc), the
- * partial top-k lists live in one statically sized device array of 16 MiB
- * that the library holds on every GPU that loads it until the process exits.
- *   - A search whose lists need more than 16 MiB (many queries with a large
- *     k, e.g. k > 32 over thousands of queries) is refused with
+ * Same arguments, results and stream semantics as oprag_search, and the same
+ * kernels (including the sampled first pass of k > 32 over a large corpus).
+ * Instead of the index's scratch buffer (which oprag_search grows with
+ * cudaMalloc), the partial top-k lists, the sampled pass and the per-query
+ * shared bounds live in one statically sized device array of 16 MiB that the
+ * library holds on every GPU that loads it until the process exits.
+ *   - A search that needs more than 16 MiB (many queries with a large k,
+ *     e.g. k > 32 over thousands of queries) is refused with
  *     OPRAG_ERR_INVALID_ARG and a message giving the required size; nothing
  *     is launched.
  *   - The first call on a device resolves the array's device address (a
- *     runtime query, no allocation); make that first call before any stream
- *     capture.
+ *     runtime query, no allocation) and keeps it for the process; make that
+ *     first call before any stream capture.  A cudaDeviceReset invalidates
+ *     the kept address: do not call this entry point after one.
  *   - All calls share the array, so calls that overlap on the GPU (different
  *     indexes or streams without ordering between them) race; order them.
- *     The kernels initialise every list they use, so nothing from an earlier
- *     call leaks into a later one.
+ *     The kernels initialise every list they use and each call clears its
+ *     shared bounds, so nothing from an earlier call leaks into a later one.
+ *   - With timing on (OPRAG_OPT_TIMING) it records the same events as
+ *     oprag_search.
  */
 OPRAG_API int oprag_search_noalloc(oprag_index *idx, const void *queries, int32_t q, int32_t k,
                                    int64_t *out_ids, float *out_scores, void *stream);

@@ -93,3 +93,19 @@ def check_topk(gpu_ids, gpu_scores, or_ids, or_scores, k: int, tol: float = 1e-4
             e = abs(float(gpu_scores[i][r]) - float(or_scores[i][pos[int(gpu_ids[i][r])]]))
             max_err = max(max_err, e)
     return {"queries": q, "exact_id_lists": exact, "max_abs_score_err": max_err}
+
+
+def topk_with_margin(fn, k: int, n: int, tol: float = 1e-4, margin: int = 48):
+    """Calls fn(kout) -> (ids, scores, ...) with kout = k + margin ranks of the
+    oracle, growing the margin until the near-tie block at rank k ends inside
+    the returned ranks for every row (or every chunk is returned)."""
+    while True:
+        kout = min(n, k + margin)
+        res = fn(kout)
+        ids, sc = res[0], res[1]
+        if kout >= n:
+            return ids, sc
+        if all(near_tie_blocks(sc[i], tol)[-1] != near_tie_blocks(sc[i], tol)[k - 1]
+               for i in range(sc.shape[0])):
+            return ids, sc
+        margin *= 4

@@ -18,6 +18,7 @@ OPRAG_OPT_TIMING = 3
 OPRAG_OPT_PAIR = 4
 OPRAG_OPT_BOUND_TAG = 5
 OPRAG_OPT_GRAPH = 6
+OPRAG_OPT_WAIT_LIMIT = 7
 
 ERRORS = {
     0: "OK",
@@ -62,7 +63,9 @@ SIGNATURES = {
     "oprag_plan_search": (_I32, [ctypes.c_int64, _I32, _I32, _I32, _I32, _I32, _I32, _I32,
                                  ctypes.POINTER(ctypes.c_int64)]),
     "oprag_index_last_timing": (_I32, [_P, ctypes.POINTER(_F), ctypes.POINTER(_F),
-                                       ctypes.POINTER(_F)]),
+                                       ctypes.POINTER(_F), ctypes.POINTER(_F)]),
+    "oprag_index_buffer_bytes": (_I32, [_P, ctypes.POINTER(_I64), ctypes.POINTER(_I64),
+                                        ctypes.POINTER(_I64)]),
     "oprag_last_error": (ctypes.c_char_p, []),
 }
 

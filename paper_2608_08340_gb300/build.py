@@ -18,6 +18,8 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(OUT_DIR, "liboprag.so")
+# The nvcc command lines of the last build, one per line (compiles, then the link).
+COMMANDS_PATH = os.path.join(OUT_DIR, "nvcc_commands.txt")
 
 ARCH = "-gencode=arch=compute_103a,code=sm_103a"
 
@@ -73,6 +75,8 @@ def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | N
             print(r.stderr)
         return obj
 
+    commands = [[nvcc, "-c", src, "-o", os.path.join(OUT_DIR, os.path.basename(src) + ".o")]
+                + flags for src in sources()]
     with cf.ThreadPoolExecutor(max_workers=max(1, min(8, os.cpu_count() or 1))) as ex:
         objs = list(ex.map(compile_one, sources()))
     libdir = _cuda_lib_dir(nvcc)
@@ -82,6 +86,9 @@ def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | N
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stderr}")
+    with open(COMMANDS_PATH, "w") as f:
+        for c in commands + [cmd]:
+            f.write(" ".join(c) + "\n")
     os.replace(tmp, LIB_PATH)
     return LIB_PATH
 

@@ -372,16 +372,16 @@ __device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
 }
 
 // Waits for the phase with the given parity to complete.  Gives up when the
-// CTA-wide abort word is set or the cycle limit passes (then sets both).
+// CTA-wide abort word is set or `limit` cycles pass (then sets both).
 template <bool kCluster = false>
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                          int* dev_err) {
+                                          int* dev_err, long long limit = kWaitLimitCycles) {
   if (mbar_test<kCluster>(bar, parity)) return true;
   const long long t0 = clock64();
   while (true) {
     if (mbar_test<kCluster>(bar, parity)) return true;
     if (*abort_flag) return false;
-    if (clock64() - t0 > kWaitLimitCycles) {
+    if (clock64() - t0 > limit) {
       *abort_flag = 1;
       atomicExch(dev_err, static_cast<int>(kDevErrWaitTimeout));
       return false;

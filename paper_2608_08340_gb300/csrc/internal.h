@@ -91,11 +91,14 @@ size_t tc_scratch_bytes(const SearchShape& s, const TcPlan& p);
 // levels / level_cnt (optional, q x kLevels, buffered lists only): candidate
 // floors and zeroed counters; a floor becomes a shared bound once k pushed
 // keys reach it.
+// wait_limit: cycles an mbarrier wait may spin before the kernel gives up and
+// sets *dev_err (<= 0: the default of about a second).
 cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s, const Fusion& fu,
                              const TcPlan& plan, void* scratch, int* dev_err, ListSet* lists,
                              cudaStream_t st, const float* init_floor = nullptr,
                              uint64_t* qfloor = nullptr, uint32_t gen = 0,
-                             const float* levels = nullptr, int* level_cnt = nullptr);
+                             const float* levels = nullptr, int* level_cnt = nullptr,
+                             long long wait_limit = 0);
 
 // --- final merge of partial lists into the sorted top-k per query.
 // kth_out (optional, q floats): the k-th best merged score of every query

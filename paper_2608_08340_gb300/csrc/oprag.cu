@@ -125,12 +125,17 @@ struct oprag_index {
   int last_grid = 0, last_cluster = 0, last_block_n = 0;   // last main search kernel launch
   int last_tiles = 0;                                         // query tiles per CTA and unit
 
-  // Optional kernel timing: events before the lexical pass, before the
-  // search kernel, before the merge kernel and after it.
+  // Optional kernel timing (events listed below).
   bool timing = false;
   bool timed = false;      // the last search recorded its events
   bool timed_lex = false;  // ... including a lexical pass
-  cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
+  bool timed_sample = false;  // ... including a sampled first pass
+  // ev[0] before the lexical pass, ev[1] before the search passes, ev[4]
+  // before the main search pass (after the sampled first pass, if any),
+  // ev[2] before the merge, ev[3] after it.
+  cudaEvent_t ev[5] = {nullptr, nullptr, nullptr, nullptr, nullptr};
+  // Spin limit (cycles) of the search kernels' mbarrier waits; 0 = default.
+  long long wait_limit = 0;
 
   // Waits until all work enqueued on this index is done.
   cudaError_t drain() { return done ? cudaEventSynchronize(done) : cudaSuccess; }
@@ -242,87 +247,123 @@ int choose_path(const oprag_index* idx, int q) {
   return q <= kSimtMaxQueriesBf16 ? 1 : 2;
 }
 
-// Dense (or fused) top-k of q queries; all pointers on the device.
-int run_search(oprag_index* idx, const void* Q, int q, int k, const Fusion& fu, int64_t* out_ids,
-               float* out_scores, cudaStream_t st) {
+// Scratch of one search, in one block: the main pass's partial lists and,
+// for buffered lists (k > 32) over many corpus tiles, a first pass over every
+// kSampleStride-th corpus tile (its lists, its merged top-k, and per query the
+// k-th score, kLevels counted floors and their counters).  Register lists
+// (k <= 32) also use one 64-bit shared bound per query, kept outside the block.
+constexpr int kSampleStride = 16;
+
+struct SearchLayout {
+  int path = 0;           // 1 SIMT, 2 tensor core
+  int simt_grid = 0;
+  TcPlan plan{}, splan{};
+  bool sampled = false;
+  size_t main_bytes = 0;    // multiple of 256
+  size_t sample_bytes = 0;  // 0 unless sampled
+  bool floors = false;      // q shared bounds (register lists on the tensor-core path)
+  size_t total() const { return main_bytes + sample_bytes; }
+};
+
+size_t round256(size_t b) { return (b + 255) / 256 * 256; }
+
+SearchLayout search_layout(oprag_index* idx, int q, int k, int path, int block_n, int pair) {
+  SearchLayout L;
   SearchShape s{idx->n, idx->d, q, k};
-  const int path = choose_path(idx, q);
-  ListSet lists{};
-  TcPlan plan_used{};
-  cudaError_t e;
+  L.path = path;
   if (path == 1) {
-    const int grid = simt_grid(s, idx->num_sms);
-    int rc = idx->ensure(&idx->scratch, &idx->scratch_bytes, simt_scratch_bytes(idx->dtype, s, grid),
-                         "search scratch");
-    if (rc) return rc;
-    if (idx->timing) cudaEventRecord(idx->ev[1], st);
-    e = launch_simt_search(idx->dtype, idx->emb, Q, s, fu, idx->scratch, grid, &lists, st);
-  } else {
-    const TcPlan plan = tc_plan(s, idx->num_sms, idx->opt_block_n, 1, idx->opt_pair, pair_capacity(idx));
-    const size_t main_bytes = (tc_scratch_bytes(s, plan) + 255) / 256 * 256;
-    // Buffered lists (k > 32) collect every score above their floor, and the
-    // floor of a fresh list starts at -inf.  A cheap first pass over every
-    // kSampleStride-th corpus tile with 32-key lists yields, per query, the
-    // k-th best of real corpus scores -- a lower bound of the true k-th best
-    // -- which the main pass then uses as the lists' starting floor.
-    constexpr int kSampleStride = 16;
-    const bool sampled = list_len_for(k) > 32 && plan.nt >= 8 * kSampleStride;
+    L.simt_grid = simt_grid(s, idx->num_sms);
+    L.main_bytes = round256(simt_scratch_bytes(idx->dtype, s, L.simt_grid));
+    return L;
+  }
+  L.plan = tc_plan(s, idx->num_sms, block_n, 1, pair, pair_capacity(idx));
+  L.main_bytes = round256(tc_scratch_bytes(s, L.plan));
+  // Buffered lists collect every score above their floor, and the floor of a
+  // fresh list starts at -inf.  A cheap first pass over every
+  // kSampleStride-th corpus tile with 32-key lists yields, per query, the
+  // k-th best of real corpus scores -- a lower bound of the true k-th best --
+  // which the main pass then uses as the lists' starting floor.
+  L.sampled = list_len_for(k) > 32 && L.plan.nt >= 8 * kSampleStride;
+  if (L.sampled) {
     SearchShape s32 = s;
     s32.k = 32;
-    TcPlan splan{};
-    size_t sample_bytes = 0;
-    // Sampled-pass scratch: its lists, its merged top-k (ids + scores), then
-    // per query the k-th score, kLevels counted floors and their counters.
+    L.splan = tc_plan(s32, idx->num_sms, L.plan.block_n, kSampleStride, L.plan.pair,
+                      pair_capacity(idx));
     const size_t per_query_tail = sizeof(float) + kLevels * (sizeof(float) + sizeof(int));
-    if (sampled) {
-      splan = tc_plan(s32, idx->num_sms, plan.block_n, kSampleStride, plan.pair, pair_capacity(idx));
-      sample_bytes = (tc_scratch_bytes(s32, splan) + 255) / 256 * 256 +
-                     (static_cast<size_t>(q) * k * 12 + 255) / 256 * 256 +
+    L.sample_bytes = round256(tc_scratch_bytes(s32, L.splan)) +
+                     round256(static_cast<size_t>(q) * k * 12) +
                      static_cast<size_t>(q) * per_query_tail + 16;
-    }
-    int rc = idx->ensure(&idx->scratch, &idx->scratch_bytes, main_bytes + sample_bytes,
-                         "search scratch");
-    if (rc) return rc;
-    if (idx->timing) cudaEventRecord(idx->ev[1], st);
+  }
+  L.floors = list_len_for(k) <= 32;
+  return L;
+}
+
+SearchLayout search_layout(oprag_index* idx, int q, int k) {
+  return search_layout(idx, q, k, choose_path(idx, q), idx->opt_block_n, idx->opt_pair);
+}
+
+// Enqueues the passes of a laid-out search and its merge.  scratch holds
+// L.total() bytes; qf / gen are the shared bounds (used when L.floors).
+int launch_search(oprag_index* idx, const SearchLayout& L, const void* Q, int q, int k,
+                  const Fusion& fu, void* scratch, uint64_t* qf, uint32_t gen, int64_t* out_ids,
+                  float* out_scores, cudaStream_t st) {
+  SearchShape s{idx->n, idx->d, q, k};
+  ListSet lists{};
+  cudaError_t e;
+  if (idx->timing) cudaEventRecord(idx->ev[1], st);
+  idx->timed_sample = idx->timing && L.sampled;
+  if (L.path == 1) {
+    e = launch_simt_search(idx->dtype, idx->emb, Q, s, fu, scratch, L.simt_grid, &lists, st);
+  } else {
     const float* floor = nullptr;
     float* levels = nullptr;
     int* level_cnt = nullptr;
-    if (sampled) {
-      char* sbase = static_cast<char*>(idx->scratch) + main_bytes;
-      const size_t slist = (tc_scratch_bytes(s32, splan) + 255) / 256 * 256;
+    if (L.sampled) {
+      SearchShape s32 = s;
+      s32.k = 32;
+      char* sbase = static_cast<char*>(scratch) + L.main_bytes;
+      const size_t slist = round256(tc_scratch_bytes(s32, L.splan));
       int64_t* sids = reinterpret_cast<int64_t*>(sbase + slist);
       float* sscores = reinterpret_cast<float*>(sids + static_cast<size_t>(q) * k);
-      float* kth = reinterpret_cast<float*>(
-          sbase + slist + (static_cast<size_t>(q) * k * 12 + 255) / 256 * 256);
+      float* kth = reinterpret_cast<float*>(sbase + slist + round256(static_cast<size_t>(q) * k * 12));
       // 16-byte aligned: each query's kLevels counters are read as one int4.
       levels = kth + (static_cast<size_t>(q) + 3) / 4 * 4;
       level_cnt = reinterpret_cast<int*>(levels + static_cast<size_t>(q) * kLevels);
       ListSet slists{};
-      e = launch_tc_search(idx->emb, Q, s32, fu, splan, sbase, idx->dev_err, &slists, st);
+      e = launch_tc_search(idx->emb, Q, s32, fu, L.splan, sbase, idx->dev_err, &slists, st,
+                           nullptr, nullptr, 0, nullptr, nullptr, idx->wait_limit);
       if (e == cudaSuccess) e = launch_merge(slists, q, k, sids, sscores, st, kth, levels);
       if (e == cudaSuccess)
         e = cudaMemsetAsync(level_cnt, 0, static_cast<size_t>(q) * kLevels * sizeof(int), st);
       if (e != cudaSuccess) return cuda_fail(e, "sampling pass");
       floor = kth;
     }
-    uint64_t* qf = nullptr;
-    uint32_t gen = 0;
-    if (list_len_for(k) <= 32) {
-      if ((rc = shared_floors(idx, q, st, &qf, &gen))) return rc;
-    }
-    e = launch_tc_search(idx->emb, Q, s, fu, plan, idx->scratch, idx->dev_err, &lists, st, floor,
-                         qf, gen, levels, level_cnt);
-    plan_used = plan;
+    if (idx->timed_sample) cudaEventRecord(idx->ev[4], st);
+    e = launch_tc_search(idx->emb, Q, s, fu, L.plan, scratch, idx->dev_err, &lists, st, floor,
+                         L.floors ? qf : nullptr, gen, levels, level_cnt, idx->wait_limit);
   }
   if (e != cudaSuccess) return cuda_fail(e, "search kernel");
   if (idx->timing) cudaEventRecord(idx->ev[2], st);
-  note_launch(idx, path, plan_used);
+  note_launch(idx, L.path, L.plan);
   e = launch_merge(lists, q, k, out_ids, out_scores, st);
   if (e != cudaSuccess) return cuda_fail(e, "merge kernel");
   if (idx->timing) cudaEventRecord(idx->ev[3], st);
   idx->timed = idx->timing;
-  idx->last_path = path;
+  idx->last_path = L.path;
   return OPRAG_OK;
+}
+
+// Dense (or fused) top-k of q queries; all pointers on the device.  Grows the
+// index's scratch (and shared bounds) on demand.
+int run_search(oprag_index* idx, const void* Q, int q, int k, const Fusion& fu, int64_t* out_ids,
+               float* out_scores, cudaStream_t st) {
+  const SearchLayout L = search_layout(idx, q, k);
+  int rc = idx->ensure(&idx->scratch, &idx->scratch_bytes, L.total(), "search scratch");
+  if (rc) return rc;
+  uint64_t* qf = nullptr;
+  uint32_t gen = 0;
+  if (L.floors && (rc = shared_floors(idx, q, st, &qf, &gen))) return rc;
+  return launch_search(idx, L, Q, q, k, fu, idx->scratch, qf, gen, out_ids, out_scores, st);
 }
 
 int check_search_args(const oprag_index* idx, const void* queries, int q, int k,
@@ -480,21 +521,34 @@ int oprag_index_reserve(oprag_index* idx, int32_t q_max, int32_t k_max) {
   if (q_max < 1 || k_max < 1 || k_max > OPRAG_K_MAX)
     return fail(OPRAG_ERR_INVALID_ARG, "bad reservation q_max=%d k_max=%d", q_max, k_max);
   DeviceGuard g(idx->device);
-  SearchShape s{idx->n, idx->d, q_max, std::min<int>(k_max, static_cast<int>(std::min<int64_t>(idx->n, OPRAG_K_MAX)))};
-  size_t need = simt_scratch_bytes(idx->dtype, s, simt_grid(s, idx->num_sms));
-  if (idx->dtype == OPRAG_BF16) {
-    for (int bn : {64, 256}) {
-      for (int qq : {q_max, std::min(q_max, 128)}) {
-        SearchShape s2 = s;
-        s2.q = qq;
-        for (int pair : {1, 2, 3})
-          need = std::max(need, tc_scratch_bytes(s2, tc_plan(s2, idx->num_sms, bn, 1, pair,
-                                                             pair_capacity(idx))));
-      }
+  const int kcap = static_cast<int>(std::min<int64_t>({k_max, idx->n, OPRAG_K_MAX}));
+  // Every layout a search of up to q_max queries and k_max results may take:
+  // each list length up to k_max's, both kernel families, every forced tile
+  // width and CTA mode, and a single query tile (whose plan differs).
+  size_t need = 0;
+  for (int kk : {8, 16, 32, 128, 256}) {
+    const int k = std::min(kk, kcap);
+    for (int qq : {static_cast<int>(q_max), std::min<int>(q_max, 128)}) {
+      need = std::max(need, search_layout(idx, qq, k, 1, 0, 0).total());
+      if (idx->dtype != OPRAG_BF16) continue;
+      for (int bn : {0, 128, 256})
+        for (int pair : {0, 1, 2, 3})
+          need = std::max(need, search_layout(idx, qq, k, 2, bn, pair).total());
     }
   }
   int rc = idx->ensure(&idx->scratch, &idx->scratch_bytes, need, "search scratch");
   if (rc) return rc;
+  // Shared k-th bounds of register lists: zeroed once here, so that a later
+  // search of up to q_max queries neither allocates nor clears them.
+  const size_t fb = static_cast<size_t>(q_max) * sizeof(uint64_t);
+  if (fb > idx->qfloor_bytes) {
+    rc = idx->ensure(reinterpret_cast<void**>(&idx->qfloor), &idx->qfloor_bytes, fb,
+                     "shared k-th score bounds");
+    if (rc) return rc;
+    cudaError_t e = cudaMemset(idx->qfloor, 0, idx->qfloor_bytes);
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(e, "clearing shared bounds");
+  }
   if (idx->has_sparse) {
     const int64_t ld = (idx->n + 3) / 4 * 4;
     const int64_t qc = std::min<int64_t>(q_max, std::max<int64_t>(1, kLexMaxElems / ld));
@@ -1078,6 +1132,11 @@ int oprag_index_set_option(oprag_index* idx, int32_t option, int32_t value) {
     idx->timing = value != 0;
     return ok();
   }
+  if (option == OPRAG_OPT_WAIT_LIMIT) {
+    if (value < 0) return fail(OPRAG_ERR_INVALID_ARG, "wait limit %d", value);
+    idx->wait_limit = value;
+    return ok();
+  }
   if (option == OPRAG_OPT_BOUND_TAG) {
     idx->gen = static_cast<uint32_t>(value);
     return ok();
@@ -1134,21 +1193,33 @@ int oprag_index_last_tiles_per_cta(const oprag_index* idx, int32_t* tiles) {
   return ok();
 }
 
-int oprag_index_last_timing(oprag_index* idx, float* lexical_ms, float* search_ms,
-                            float* merge_ms) {
+int oprag_index_last_timing(oprag_index* idx, float* lexical_ms, float* sample_ms,
+                            float* search_ms, float* merge_ms) {
   if (!idx) return fail(OPRAG_ERR_INVALID_ARG, "index is NULL");
   if (!idx->timed) return fail(OPRAG_ERR_NOT_READY, "no timed search was issued");
   DeviceGuard g(idx->device);
   cudaError_t e = cudaEventSynchronize(idx->ev[3]);
   if (e != cudaSuccess) return cuda_fail(e, "timing");
-  float a = 0.f, b = 0.f, c = 0.f;
+  float a = 0.f, b = 0.f, c = 0.f, m = 0.f;
   if (idx->timed_lex) e = cudaEventElapsedTime(&a, idx->ev[0], idx->ev[1]);
-  if (e == cudaSuccess) e = cudaEventElapsedTime(&b, idx->ev[1], idx->ev[2]);
-  if (e == cudaSuccess) e = cudaEventElapsedTime(&c, idx->ev[2], idx->ev[3]);
+  if (e == cudaSuccess && idx->timed_sample) e = cudaEventElapsedTime(&b, idx->ev[1], idx->ev[4]);
+  if (e == cudaSuccess)
+    e = cudaEventElapsedTime(&c, idx->ev[idx->timed_sample ? 4 : 1], idx->ev[2]);
+  if (e == cudaSuccess) e = cudaEventElapsedTime(&m, idx->ev[2], idx->ev[3]);
   if (e != cudaSuccess) return cuda_fail(e, "timing");
   if (lexical_ms) *lexical_ms = a;
-  if (search_ms) *search_ms = b;
-  if (merge_ms) *merge_ms = c;
+  if (sample_ms) *sample_ms = b;
+  if (search_ms) *search_ms = c;
+  if (merge_ms) *merge_ms = m;
+  return ok();
+}
+
+int oprag_index_buffer_bytes(const oprag_index* idx, int64_t* scratch, int64_t* bounds,
+                             int64_t* lexical) {
+  if (!idx) return fail(OPRAG_ERR_INVALID_ARG, "index is NULL");
+  if (scratch) *scratch = static_cast<int64_t>(idx->scratch_bytes);
+  if (bounds) *bounds = static_cast<int64_t>(idx->qfloor_bytes);
+  if (lexical) *lexical = static_cast<int64_t>(idx->lex_bytes);
   return ok();
 }
 
@@ -1176,7 +1247,9 @@ std::mutex g_static_mu;
 void* g_static_ptr[kMaxDevices] = {};
 
 // Device address of g_static_scratch on `device` (which must be current),
-// resolved once per device.  The host-side name is only a stand-in.
+// resolved once per device.  The host-side name is only a stand-in.  The
+// cached address belongs to the device's primary context: after a
+// cudaDeviceReset it is stale (the header says so).
 int static_scratch(int device, void** out) {
   if (device < 0 || device >= kMaxDevices)
     return fail(OPRAG_ERR_INVALID_ARG, "device %d out of range", device);
@@ -1202,33 +1275,27 @@ extern "C" int oprag_search_noalloc(oprag_index* idx, const void* queries, int32
   void* scratch = nullptr;
   if ((rc = static_scratch(idx->device, &scratch))) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  SearchShape s{idx->n, idx->d, q, k};
-  const int path = choose_path(idx, q);
-  size_t need;
-  TcPlan plan{};
-  int grid = 0;
-  if (path == 1) {
-    grid = simt_grid(s, idx->num_sms);
-    need = simt_scratch_bytes(idx->dtype, s, grid);
-  } else {
-    plan = tc_plan(s, idx->num_sms, idx->opt_block_n, 1, idx->opt_pair, pair_capacity(idx));
-    need = tc_scratch_bytes(s, plan);
-  }
+  // The same passes as oprag_search (with the sampled first pass for k > 32
+  // over many corpus tiles); its shared per-query bounds sit after the lists
+  // and are cleared on every call, since the array is shared by all indexes.
+  const SearchLayout L = search_layout(idx, q, k);
+  const size_t floors = L.floors ? static_cast<size_t>(q) * sizeof(uint64_t) : 0;
+  const size_t need = round256(L.total()) + floors;
   if (need > kStaticScratchBytes)
     return fail(OPRAG_ERR_INVALID_ARG,
                 "this search needs %zu bytes of scratch but the static array holds %zu; use "
                 "oprag_search or fewer queries / a smaller k",
                 need, kStaticScratchBytes);
   if ((rc = begin_call(idx, st))) return rc;
+  uint64_t* qf = nullptr;
+  if (L.floors) {
+    qf = reinterpret_cast<uint64_t*>(static_cast<char*>(scratch) + round256(L.total()));
+    cudaError_t e = cudaMemsetAsync(qf, 0, floors, st);
+    if (e != cudaSuccess) return cuda_fail(e, "clearing shared bounds");
+  }
   const Fusion none{nullptr, 0, nullptr, 0.f};
-  ListSet lists{};
-  cudaError_t e =
-      path == 1 ? launch_simt_search(idx->dtype, idx->emb, queries, s, none, scratch, grid, &lists, st)
-                : launch_tc_search(idx->emb, queries, s, none, plan, scratch, idx->dev_err, &lists, st);
-  if (e != cudaSuccess) return cuda_fail(e, "search kernel");
-  note_launch(idx, path, plan);
-  e = launch_merge(lists, q, k, out_ids, out_scores, st);
-  if (e != cudaSuccess) return cuda_fail(e, "merge kernel");
-  idx->last_path = path;
+  idx->timed_lex = false;
+  if ((rc = launch_search(idx, L, queries, q, k, none, scratch, qf, 1u, out_ids, out_scores, st)))
+    return rc;
   return end_call(idx, st);
 }

@@ -68,6 +68,9 @@ struct TcParams {
   int* meta_count;      // buffered lists: kept keys per (list, row)
   uint64_t* meta_worst; // buffered lists: K-th key per (list, row)
   int* dev_err;
+  // Cycles a wait on an mbarrier may spin before the kernel gives up
+  // (kWaitLimitCycles unless a test shortens it).
+  long long wait_limit;
   // Optional (register lists only): per query, a lower bound of its k-th best
   // score shared by every list of the search, tagged with `gen` (entries of
   // other searches read as -inf); see shared_floor_read.
@@ -713,7 +716,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             if (++s == S) { s = 0; ph ^= 1u; }
             continue;
           }
-          if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, p.dev_err)) { ok = false; break; }
+          if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag, p.dev_err, p.wait_limit)) { ok = false; break; }
           load_stage(s, kb, j, t);
           issued |= 1u << s;
           parity = (parity & ~(1u << s)) | (ph << s);
@@ -740,13 +743,13 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         if constexpr (kDual) {
           // Both accumulators of buffer acc take this unit.
           const int a0i = 2 * acc, a1i = 2 * acc + 1;
-          if (!mbar_wait(&tempty[a0i], acc_ph ^ 1u, abort_flag, p.dev_err)) break;
-          if (!mbar_wait(&tempty[a1i], acc_ph ^ 1u, abort_flag, p.dev_err)) break;
+          if (!mbar_wait(&tempty[a0i], acc_ph ^ 1u, abort_flag, p.dev_err, p.wait_limit)) break;
+          if (!mbar_wait(&tempty[a1i], acc_ph ^ 1u, abort_flag, p.dev_err, p.wait_limit)) break;
           tc_fence_after();
           const uint32_t d0 = tmem_base + static_cast<uint32_t>(a0i * BN);
           const uint32_t d1 = tmem_base + static_cast<uint32_t>(a1i * BN);
           for (int kb = 0; kb < p.kblocks; ++kb) {
-            if (!mbar_wait(&full[s], ph, abort_flag, p.dev_err)) { ok = false; break; }
+            if (!mbar_wait(&full[s], ph, abort_flag, p.dev_err, p.wait_limit)) { ok = false; break; }
             tc_fence_after();
             const uint64_t a0 = sw128_desc(smem_addr(sA + s * kAStage));
             const uint64_t a1 = sw128_desc(smem_addr(sA + s * kAStage + kAStageBytes));
@@ -766,11 +769,11 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
           if (++acc == 2) { acc = 0; acc_ph ^= 1u; }
           continue;
         }
-        if (!mbar_wait<kPair>(&tempty[acc], acc_ph ^ 1u, abort_flag, p.dev_err)) break;
+        if (!mbar_wait<kPair>(&tempty[acc], acc_ph ^ 1u, abort_flag, p.dev_err, p.wait_limit)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
         for (int kb = 0; kb < p.kblocks; ++kb) {
-          if (!mbar_wait(&full[s], ph, abort_flag, p.dev_err)) { ok = false; break; }
+          if (!mbar_wait(&full[s], ph, abort_flag, p.dev_err, p.wait_limit)) { ok = false; break; }
           tc_fence_after();
           const uint64_t a = sw128_desc(smem_addr(sA + s * kAStage));
           const uint64_t b = sw128_desc(smem_addr(sB + s * kBStageBytes));
@@ -867,7 +870,11 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       } else {
         if (act) gfl = list.proven_floor(p.k);
       }
-      if (!mbar_wait(&tfull[acc], (acc_ph >> acc) & 1u, abort_flag, p.dev_err)) break;
+      // The warp leaves together when a wait gives up: the TMEM loads below
+      // are warp-collective.
+      const bool got = mbar_wait(&tfull[acc], (acc_ph >> acc) & 1u, abort_flag, p.dev_err,
+                                 p.wait_limit);
+      if (!__all_sync(0xffffffffu, got)) break;
       tc_fence_after();
       if (warp_live) {
         float inv_max = 0.f;

@@ -220,11 +220,24 @@ class Index:
         self.set_option(_lib.OPRAG_OPT_TIMING, int(on))
 
     def last_timing(self) -> dict:
-        """Device milliseconds of the last timed search's kernels."""
-        a, b, c = ctypes.c_float(), ctypes.c_float(), ctypes.c_float()
+        """Device milliseconds of the last timed search's kernels: lexical pass,
+        sampled first pass (k > 32 over many tiles), main search pass, merge."""
+        a, b, c, m = ctypes.c_float(), ctypes.c_float(), ctypes.c_float(), ctypes.c_float()
         check(self._lib.oprag_index_last_timing(self._h, ctypes.byref(a), ctypes.byref(b),
-                                                ctypes.byref(c)))
-        return {"lexical_ms": a.value, "search_ms": b.value, "merge_ms": c.value}
+                                                ctypes.byref(c), ctypes.byref(m)))
+        return {"lexical_ms": a.value, "sample_ms": b.value, "search_ms": c.value,
+                "merge_ms": m.value}
+
+    def buffer_bytes(self) -> dict:
+        """Bytes held by the index's grow-on-demand device buffers."""
+        a, b, c = ctypes.c_int64(), ctypes.c_int64(), ctypes.c_int64()
+        check(self._lib.oprag_index_buffer_bytes(self._h, ctypes.byref(a), ctypes.byref(b),
+                                                 ctypes.byref(c)))
+        return {"scratch": a.value, "bounds": b.value, "lexical": c.value}
+
+    def set_wait_limit(self, cycles: int) -> None:
+        """Test hook: spin limit of the search kernels' barrier waits (0 = default)."""
+        self.set_option(_lib.OPRAG_OPT_WAIT_LIMIT, int(cycles))
 
     @property
     def last_launch(self) -> dict:

@@ -14,8 +14,9 @@ near ties) stand in for the embeddings, and Zipf-distributed token bags stand
 in for the chunk text that BM25 indexes.
 
 Recipe (all numpy PCG64 ``default_rng``):
-  * dense rows: float32 standard normals drawn in chunks of 65536 rows,
-    normalised in float64, cast to float32; bf16 inputs are the
+  * dense rows: float32 standard normals drawn in chunks of 65536 rows
+    (chunk c from its own generator seeded (seed, c)), normalised in float64,
+    cast to float32; bf16 inputs are the
     round-to-nearest-even bf16 of that float32 (torch ``.to(bfloat16)``).
   * clustered rows: centres ~ N(0, I); each row picks a centre uniformly;
     x = c + sigma * z; then normalised as above.
@@ -49,12 +50,26 @@ def to_bf16_bits(x32: np.ndarray) -> np.ndarray:
 
 
 def gaussian_rows(n: int, d: int, seed: int) -> np.ndarray:
-    """n x d float32 L2-normalised Gaussian directions."""
-    rng = np.random.default_rng(seed)
+    """n x d float32 L2-normalised Gaussian directions.  Rows come in chunks of
+    65536; chunk c draws from its own generator seeded (seed, c), so the
+    chunks can be drawn on several threads and the result does not depend on
+    how many."""
     out = np.empty((n, d), np.float32)
-    for lo in range(0, n, _CHUNK):
-        hi = min(n, lo + _CHUNK)
+
+    def fill(c: int) -> None:
+        lo, hi = c * _CHUNK, min(n, (c + 1) * _CHUNK)
+        rng = np.random.default_rng([seed, c])
         out[lo:hi] = _normalise(rng.standard_normal((hi - lo, d), dtype=np.float32))
+
+    chunks = range((n + _CHUNK - 1) // _CHUNK)
+    if len(chunks) <= 1:
+        for c in chunks:
+            fill(c)
+    else:
+        import concurrent.futures as cf
+        import os
+        with cf.ThreadPoolExecutor(max_workers=min(len(chunks), os.cpu_count() or 1)) as ex:
+            list(ex.map(fill, chunks))
     return out
 
 

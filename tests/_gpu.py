@@ -17,23 +17,9 @@ def dev_tensor(a: np.ndarray, device="cuda") -> torch.Tensor:
 
 
 def oracle_topk(fn, k: int, n: int, margin: int = 48):
-    """Calls fn(kout) -> (ids, scores, ...) with kout = k + margin, growing the
-    margin until the near-tie block at rank k is complete for every row."""
-    while True:
-        kout = min(n, k + margin)
-        res = fn(kout)
-        ids, sc = res[0], res[1]
-        if kout >= n:
-            return ids, sc
-        short = False
-        for i in range(sc.shape[0]):
-            blocks = check.near_tie_blocks(sc[i], TOL)
-            if blocks[-1] == blocks[k - 1]:
-                short = True
-                break
-        if not short:
-            return ids, sc
-        margin *= 4
+    """Calls fn(kout) -> (ids, scores, ...) with enough oracle ranks for the
+    near-tie rule at rank k (oracle/check.py)."""
+    return check.topk_with_margin(fn, k, n, TOL, margin)
 
 
 def check_dense(ids, scores, E_data, Q_data, k, label="", rows=None):

@@ -41,9 +41,28 @@ def test_binding_covers_every_declared_symbol():
 
 
 def test_library_targets_sm103a_only():
-    out = lib_build.build()
-    data = open(out, "rb").read()
-    assert b"sm_103a" in data or b"sm_103" in data
+    """Every nvcc command of the build (each compile and the link) names
+    sm_103a as its only target."""
+    assert lib_build.ARCH == "-gencode=arch=compute_103a,code=sm_103a"
+    lib_build.build()
+    if not os.path.exists(lib_build.COMMANDS_PATH):      # built before commands were recorded
+        lib_build.build(force=True)
+    lines = open(lib_build.COMMANDS_PATH).read().splitlines()
+    srcs = lib_build.sources()
+    assert len(lines) == len(srcs) + 1
+    for line in lines:
+        args = line.split()
+        targets = [a for a in args if "arch=" in a or a.startswith("-arch") or "code=" in a]
+        assert targets == [lib_build.ARCH], line
+    for src, line in zip(srcs, lines):
+        assert f" -c {src} " in line
+    assert " -shared " in lines[-1]
+
+
+def test_option_codes_match_header():
+    text = open(os.path.join(ROOT, "include", "oprag.h")).read()
+    for name, value in re.findall(r"#define (OPRAG_OPT_\w+) (\d+)", text):
+        assert getattr(_lib, name) == int(value), name
 
 
 def _err(lib):

@@ -167,14 +167,23 @@ def test_fp32_input_into_bf16_index_rounds_to_nearest_even():
     np.testing.assert_array_equal(got2, got)
 
 
-def test_config2_clustered_near_ties_sampled():
+def test_config2_clustered_near_ties_every_query():
+    """All 4096 queries of the clustered workload against the oracle."""
     w = workloads.config(2)
     idx = _index(w.E_data)
     ids, sc = idx.search(dev_tensor(w.Q_data), w.k)
     assert idx.last_path == "tc"
-    rows = np.random.default_rng(0).choice(w.q, 48, replace=False)
-    rows.sort()
-    check_dense(ids, sc, w.E_data, w.Q_data, w.k, "cfg2", rows=rows)
+    check_dense(ids, sc, w.E_data, w.Q_data, w.k, "cfg2")
+    idx.check()
+
+
+def _lane_quarter_rows(q, seed):
+    """Two random rows in every 32-query group (TMEM lane quarter) of every
+    128-query tile."""
+    rng = np.random.default_rng(seed)
+    return np.sort(np.concatenate([rng.choice(np.arange(lo, min(q, lo + 32)),
+                                              min(2, q - lo), replace=False)
+                                   for lo in range(0, q, 32)]))
 
 
 @pytest.mark.slow
@@ -185,7 +194,7 @@ def test_config4_scale_with_upserts_sampled():
     w = workloads.config(4, batch=8192)
     E = w.E_data.copy()
     idx = _index(E)
-    rng = np.random.default_rng(1)
+    idx.enable_timing(True)
     for b in range(4):
         if b > 0:
             up_ids, up_rows = workloads.upsert_batch(w.n, w.d, 4096, b, "bf16")
@@ -193,7 +202,12 @@ def test_config4_scale_with_upserts_sampled():
             oracle.upsert(E, up_ids, up_rows)
         Qb = w.Q_data[b * 2048:(b + 1) * 2048]
         ids, sc = idx.search(dev_tensor(Qb), w.k)
-        rows = np.sort(rng.choice(2048, 6, replace=False))
+        # the full-size path: CTA pairs, sampled first pass and counted floors
+        assert idx.last_launch["cluster"] == 2
+        assert idx.last_timing()["sample_ms"] > 0.0
+        # 128 rows: two in every lane quarter of all 16 query tiles
+        rows = _lane_quarter_rows(2048, seed=b)
+        assert len(rows) == 128
         check_dense(ids, sc, E, Qb, w.k, f"cfg4 batch {b}", rows=rows)
     # the index equals the oracle's post-upsert array
     got = idx.rows().view(torch.int16).numpy().view(np.uint16)

@@ -141,10 +141,10 @@ def cfg3():
     return w, idx
 
 
-def test_config3_hybrid_sampled(cfg3):
+def test_config3_hybrid_every_query(cfg3):
+    """All 1024 queries of the hybrid workload against the oracle."""
     w, idx = cfg3
-    rows = np.sort(np.random.default_rng(2).choice(w.q, 40, replace=False))
-    _hybrid_check(idx, w, rows, w.alpha, "cfg3")
+    _hybrid_check(idx, w, np.arange(w.q), w.alpha, "cfg3")
     assert idx.last_path == "tc"
     idx.check()
 

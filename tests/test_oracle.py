@@ -322,6 +322,20 @@ def test_embed_pool_golden_hand_worked():
     assert bits.tolist() == g["bf16_bits"]
 
 
+def test_embed_pool_golden_pooled_rows_are_the_masked_means():
+    """The fixture's pooled (pre-normalisation) rows are the exact means of
+    the unmasked tokens, and normalising them gives its normalised rows."""
+    from fractions import Fraction
+    g = load("embed_pool_2tok.json")
+    for h, m, pooled, normed in zip(g["hidden"], g["mask"], g["pooled"], g["normalised_exact"]):
+        toks = [t for t, keep in zip(h, m) if keep]
+        mean = [sum(Fraction(t[j]) for t in toks) / len(toks) for j in range(len(h[0]))]
+        assert [Fraction(x) for x in pooled] == mean
+        norm = float(sum(x * x for x in mean)) ** 0.5
+        want = [float(x) / norm if norm else 0.0 for x in mean]
+        np.testing.assert_allclose([value(x) for x in normed], want, rtol=0, atol=1e-15)
+
+
 def test_embed_pool_single_token_and_identical_tokens_are_the_normalised_token():
     rng = np.random.default_rng(7)
     h = rng.standard_normal((5, 6, 64)).astype(np.float32)

@@ -1,13 +1,15 @@
 """oprag_search_noalloc: the search entry point for callers that must not
-allocate device memory while serving (its partial lists live in a static
-16 MiB device array instead of the index's growable scratch buffer).
+allocate device memory while serving (a process whose memory pool already
+holds the GPU, or one that cannot take the device-wide synchronisation a
+cudaMalloc or cudaFree may cause).  Its partial lists, sampled first pass and
+shared bounds live in a static 16 MiB device array instead of the index's
+growable scratch buffer.
 
-Called through the C ABI and checked against oprag_search on the same inputs,
-twice in a row (the static array keeps the previous call's contents, so the
-second call checks that nothing leaks between calls).  Kept in a file that
-pytest collects last."""
-import ctypes
-
+Called through the C ABI on a fresh index, before any oprag_search, and
+checked against oprag_search on the same inputs, twice in a row (the static
+array keeps the previous call's contents, so the second call checks that
+nothing leaks between calls); the index's own buffers must still be empty
+after the no-allocation calls.  Kept in a file that pytest collects last."""
 import numpy as np
 import pytest
 import torch
@@ -29,18 +31,29 @@ def _noalloc(lib, idx, Q, k):
     return rc, ids, sc
 
 
+# (cfg, q, k, n): dual mode (256 queries), one query, single CTAs with lists of
+# 16, the fp32 SIMT kernel, and two k > 32 cases: a small corpus (no sampled
+# pass) and 157 corpus tiles (the sampled first pass and counted floors run).
 @pytest.mark.parametrize("cfg,q,k,n", [(1, 256, 5, 20000), (1, 1, 5, 20000), (2, 300, 10, 20000),
-                                       (0, 16, 5, None), (1, 64, 100, 2000)])
+                                       (0, 16, 5, None), (1, 64, 100, 2000),
+                                       (1, 64, 100, 20000)])
 def test_noalloc_matches_search_twice(cfg, q, k, n):
     lib = _lib.load()
     w = workloads.config(cfg, batch=q, n=n)
     idx = Index(dev_tensor(w.E_data))
     Q = dev_tensor(w.Q_data)
-    ref_ids, ref_sc = idx.search(Q, k)
+    got = []
     for _ in range(2):
         rc, ids, sc = _noalloc(lib, idx, Q, k)
         assert rc == 0, lib.oprag_last_error().decode()
         torch.cuda.synchronize()
+        got.append((ids, sc))
+    # nothing was allocated for the index: its grow-on-demand buffers are empty
+    assert idx.buffer_bytes() == {"scratch": 0, "bounds": 0, "lexical": 0}
+    idx.check()
+    ref_ids, ref_sc = idx.search(Q, k)
+    torch.cuda.synchronize()
+    for ids, sc in got:
         assert torch.equal(ids, ref_ids)
         assert (sc - ref_sc).abs().max().item() <= TOL
     idx.check()
@@ -55,5 +68,6 @@ def test_noalloc_refuses_searches_beyond_the_static_array():
     assert rc == -1
     msg = lib.oprag_last_error().decode()
     assert "static array" in msg
+    torch.cuda.synchronize()
     assert (ids == -7).all()            # nothing was launched
     idx.close()
