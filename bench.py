@@ -86,6 +86,12 @@ def parse(argv=None):
                    help="measure this workload alone (default: the scale workload as the "
                         "headline plus every other workload under \"configs\")")
     p.add_argument("--batch", type=int, default=None, help="queries per step (with --config)")
+    p.add_argument("--n", type=int, default=None,
+                   help="corpus rows (with --config; a smaller case of the same kernels, e.g. "
+                        "for a profiler capture)")
+    p.add_argument("--phases", action="store_true",
+                   help="also record per-CTA global-timer stamps of the main search pass and "
+                        "report their spread (\"phases\")")
     p.add_argument("--no-cpu-baseline", action="store_true",
                    help="skip the oracle leg (parity of the timed outputs and cpu_baseline)")
     p.add_argument("--block-n", type=int, default=0, help="tensor-core tile rows (0 = auto)")
@@ -364,7 +370,7 @@ def _to_pinned(a):
 
 
 def measure(args, cfg: int, batch: int, rank: int, world: int, local_rank: int,
-            dense_first: int = 0):
+            dense_first: int = 0, n: int | None = None):
     """Times one workload on this rank's GPU.  Returns (result, w, extra) on
     rank 0 (None elsewhere); extra holds the last timed step's outputs and
     what the oracle leg needs to rebuild the index it searched."""
@@ -373,7 +379,7 @@ def measure(args, cfg: int, batch: int, rank: int, world: int, local_rank: int,
 
     dev = torch.device("cuda", local_rank)
     dense_first = dense_first if cfg == 3 else 0
-    w = workloads.config(cfg, batch=batch)
+    w = workloads.config(cfg, batch=batch, n=n)
     idx = Index(_to_dev(w.E_data, dev))
     if cfg == 3:
         idx.set_sparse(w.doc_indptr, w.doc_terms, w.vocab, w.k1, w.b)
@@ -472,6 +478,8 @@ def measure(args, cfg: int, batch: int, rank: int, world: int, local_rank: int,
             tim[key].append(t[key])
     idx.enable_timing(False)
     idx.check()
+
+    phases = phase_breakdown(idx, step, flush, min(args.steps, 20)) if args.phases else None
 
     # Warm-L2 figure, reported beside the flushed one: the same steps back to
     # back with no flush in between (a corpus under 129 MB stays in L2).
@@ -579,7 +587,7 @@ def measure(args, cfg: int, batch: int, rank: int, world: int, local_rank: int,
     roof["kernel_ms_median"] = statistics.median(tim["search_ms"])
     roof["merge_ms_mean"] = statistics.mean(tim["merge_ms"])
     if sampled:
-        # k > 32: the first pass over every 16th corpus tile and its merge,
+        # k > 32: the first pass over every 32nd corpus tile and its merge,
         # timed apart from the main pass (the dominant kernel above)
         roof["sample_pass_ms_mean"] = statistics.mean(tim["sample_ms"])
     if cfg == 3 and not dense_first:
@@ -625,16 +633,52 @@ def measure(args, cfg: int, batch: int, rank: int, world: int, local_rank: int,
                             "GB_per_s": ub / (statistics.median(upsert_ms) * 1e-3) / 1e9}
     if quality:
         result["quality"] = quality
+    if phases:
+        result["phases"] = phases
     extra = {"ids": out_ids, "scores": out_scores,
              "upserts": ([(ups[r][0], ups[r][1]) for r in upsert_sequence(args.warmup, args.steps)]
                          if cfg == 4 else [])}
     return result, w, extra
 
 
+def phase_breakdown(idx, step, flush, n_steps: int) -> dict:
+    """Per-CTA global-timer stamps of the main search pass over n_steps
+    flushed steps: for each mark, the earliest, median and latest CTA in
+    microseconds after the earliest CTA entry (median over the steps), next
+    to the same steps' event-timed kernel duration."""
+    idx.enable_phases(True)
+    idx.enable_timing(True)
+    per = {name: [] for name in idx.PHASES}
+    ev = []
+    for i in range(n_steps):
+        flush.zero_()
+        step(i)
+        ev.append(idx.last_timing()["search_ms"] * 1e3)
+        st = idx.last_phases()
+        t0 = st[:, 0][st[:, 0] > 0].min()
+        for m, name in enumerate(idx.PHASES):
+            col = st[:, m]
+            col = col[col > 0]
+            if col.size:
+                rel = (col - t0) / 1e3
+                per[name].append((float(rel.min()), float(np.median(rel)), float(rel.max())))
+    idx.enable_phases(False)
+    idx.enable_timing(False)
+    out = {"unit": "us after the first CTA entry (global timer); min / median / max over CTAs, "
+                   "median over steps",
+           "steps": n_steps, "ctas": int(st.shape[0]),
+           "kernel_event_us_median": float(np.median(ev))}
+    for name, v in per.items():
+        if v:
+            a = np.asarray(v)
+            out[name] = [round(float(np.median(a[:, c])), 2) for c in range(3)]
+    return out
+
+
 def sub_entry(res: dict) -> dict:
     """The fields of a workload's line kept under the headline's "configs"."""
     keep = ("value", "unit", "ms_per_step", "ms_per_step_median", "roofline", "e2e", "clocks",
-            "warm_l2", "parity", "gpu_launches", "path", "launch", "upsert", "metric")
+            "warm_l2", "parity", "gpu_launches", "path", "launch", "upsert", "metric", "phases")
     out = {k: res[k] for k in keep if k in res}
     out["workload"] = res["config"]["workload"]
     return out
@@ -908,7 +952,8 @@ def main():
     subs = {}
     for n_run, (cfg, batch) in enumerate(plan):
         res = measure(args, cfg, batch, rank, world, local_rank,
-                      dense_first=args.dense_first if n_run == 0 else 0)
+                      dense_first=args.dense_first if n_run == 0 else 0,
+                      n=args.n if args.config is not None else None)
         if res is None:
             continue
         result, w, extra = res

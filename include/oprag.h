@@ -293,10 +293,29 @@ OPRAG_API int oprag_index_set_option(oprag_index *idx, int32_t option, int32_t v
  * the waits of a real search run out. */
 #define OPRAG_OPT_WAIT_LIMIT 7
 
+/* OPRAG_OPT_PHASES (measurement hook): 1 makes the main tensor-core pass of
+ * every later search record, per CTA, the GPU global timer (nanoseconds) at
+ * eight points of its run; oprag_index_last_phases() reads them.  Costs one
+ * store per pipeline stage while on.  0 (default) off. */
+#define OPRAG_OPT_PHASES 8
+
+/*
+ * Global-timer stamps (ns) of the last tensor-core main pass run with
+ * OPRAG_OPT_PHASES on: *ctas receives its grid size; out (host, room for
+ * cap >= *ctas * 8 values; NULL to ask the size only) receives, per CTA, in
+ * order: entry, end of set-up (barriers, tensor memory), first pipeline
+ * stage landed, last stage landed, last MMA committed (these three only on
+ * the CTA that issues the MMAs), epilogue set 0 done, epilogue set 1 done
+ * (0 with one set), exit.  Waits for the index's pending work.
+ * OPRAG_ERR_NOT_READY when no such search ran.
+ */
+OPRAG_API int oprag_index_last_phases(oprag_index *idx, int64_t *out, int32_t cap,
+                                      int32_t *ctas);
+
 /*
  * Device durations (milliseconds) of the kernels of the last search issued
  * with timing on: lexical_ms (BM25 pass of a hybrid search, 0 for a dense
- * search), sample_ms (the first pass over every 16th corpus tile and its
+ * search), sample_ms (the first pass over every 32nd corpus tile and its
  * merge that a search with k > 32 over a large corpus runs first, else 0),
  * search_ms (main pass: score contraction + fused selection), merge_ms
  * (final top-k reduction).  Waits for that search to finish.  Any
@@ -357,10 +376,12 @@ OPRAG_API int oprag_plan_search(int64_t n, int32_t d, int32_t q, int32_t k, int3
  * cudaMalloc), the partial top-k lists, the sampled pass and the per-query
  * shared bounds live in one statically sized device array of 16 MiB that the
  * library holds on every GPU that loads it until the process exits.
- *   - A search that needs more than 16 MiB (many queries with a large k,
- *     e.g. k > 32 over thousands of queries) is refused with
+ *   - A search that needs more than 16 MiB is refused with
  *     OPRAG_ERR_INVALID_ARG and a message giving the required size; nothing
- *     is launched.
+ *     is launched.  That covers k > 32 over thousands of queries and, since
+ *     every CTA then keeps a 128-row list of 256 keys (256 KiB), k > 32 over
+ *     a corpus of 128 or more tiles of 128 chunks: the searches for which
+ *     oprag_search runs its sampled first pass.
  *   - The first call on a device resolves the array's device address (a
  *     runtime query, no allocation) and keeps it for the process; make that
  *     first call before any stream capture.  A cudaDeviceReset invalidates

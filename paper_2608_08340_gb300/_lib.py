@@ -19,6 +19,7 @@ OPRAG_OPT_PAIR = 4
 OPRAG_OPT_BOUND_TAG = 5
 OPRAG_OPT_GRAPH = 6
 OPRAG_OPT_WAIT_LIMIT = 7
+OPRAG_OPT_PHASES = 8
 
 ERRORS = {
     0: "OK",
@@ -66,6 +67,7 @@ SIGNATURES = {
                                        ctypes.POINTER(_F), ctypes.POINTER(_F)]),
     "oprag_index_buffer_bytes": (_I32, [_P, ctypes.POINTER(_I64), ctypes.POINTER(_I64),
                                         ctypes.POINTER(_I64)]),
+    "oprag_index_last_phases": (_I32, [_P, ctypes.POINTER(_I64), _I32, ctypes.POINTER(_I32)]),
     "oprag_last_error": (ctypes.c_char_p, []),
 }
 

@@ -54,19 +54,29 @@ def _stale() -> bool:
     return any(os.path.getmtime(p) > built for p in deps)
 
 
-def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | None = None) -> str:
-    """Compiles and links liboprag.so; returns its path."""
+def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | None = None,
+          out_dir: str | None = None) -> str:
+    """Compiles and links liboprag.so (into out_dir, default the in-tree
+    _build/); returns its path."""
+    if out_dir is not None and os.path.abspath(out_dir) != OUT_DIR:
+        return _build_into(os.path.abspath(out_dir), verbose, extra_flags)
     if not force and not _stale():
         return LIB_PATH
+    return _build_into(OUT_DIR, verbose, extra_flags)
+
+
+def _build_into(out_dir: str, verbose: bool, extra_flags: list[str] | None) -> str:
+    lib_path = os.path.join(out_dir, "liboprag.so")
+    commands_path = os.path.join(out_dir, "nvcc_commands.txt")
     nvcc = _nvcc()
-    os.makedirs(OUT_DIR, exist_ok=True)
+    os.makedirs(out_dir, exist_ok=True)
     flags = ["-O3", "-std=c++17", "-lineinfo", ARCH, "-Xcompiler", "-fPIC,-fvisibility=hidden",
              "-I", INCLUDE, "--expt-relaxed-constexpr"] + list(extra_flags or [])
     if verbose:
         flags += ["-Xptxas", "-v"]
 
     def compile_one(src: str) -> str:
-        obj = os.path.join(OUT_DIR, os.path.basename(src) + ".o")
+        obj = os.path.join(out_dir, os.path.basename(src) + ".o")
         cmd = [nvcc, "-c", src, "-o", obj] + flags
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
@@ -75,22 +85,22 @@ def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | N
             print(r.stderr)
         return obj
 
-    commands = [[nvcc, "-c", src, "-o", os.path.join(OUT_DIR, os.path.basename(src) + ".o")]
+    commands = [[nvcc, "-c", src, "-o", os.path.join(out_dir, os.path.basename(src) + ".o")]
                 + flags for src in sources()]
     with cf.ThreadPoolExecutor(max_workers=max(1, min(8, os.cpu_count() or 1))) as ex:
         objs = list(ex.map(compile_one, sources()))
     libdir = _cuda_lib_dir(nvcc)
-    tmp = LIB_PATH + f".tmp{os.getpid()}"
+    tmp = lib_path + f".tmp{os.getpid()}"
     cmd = [nvcc, "-shared", ARCH, "-o", tmp] + objs + [
         "-cudart", "shared", "-Xlinker", f"-rpath={libdir}"]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stderr}")
-    with open(COMMANDS_PATH, "w") as f:
+    with open(commands_path, "w") as f:
         for c in commands + [cmd]:
             f.write(" ".join(c) + "\n")
-    os.replace(tmp, LIB_PATH)
-    return LIB_PATH
+    os.replace(tmp, lib_path)
+    return lib_path
 
 
 if __name__ == "__main__":

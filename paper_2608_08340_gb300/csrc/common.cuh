@@ -371,11 +371,51 @@ __device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// Non-blocking probe of a phase (mbarrier.test_wait returns at once, where
+// try_wait may suspend the thread until the phase completes).
+template <bool kCluster = false>
+__device__ __forceinline__ bool mbar_probe(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  if constexpr (kCluster) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_addr(bar)), "r"(parity)
+        : "memory");
+  } else {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_addr(bar)), "r"(parity)
+        : "memory");
+  }
+  return ok != 0;
+}
+
 // Waits for the phase with the given parity to complete.  Gives up when the
-// CTA-wide abort word is set or `limit` cycles pass (then sets both).
+// CTA-wide abort word is set or `limit` cycles pass (then sets both).  A limit
+// below the default (a test shortening it) spins on non-blocking probes, so
+// that even a wait that hardware would complete within its suspend time runs
+// out.
 template <bool kCluster = false>
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
                                           int* dev_err, long long limit = kWaitLimitCycles) {
+  if (limit < kWaitLimitCycles) {
+    const long long t0 = clock64();
+    while (!mbar_probe<kCluster>(bar, parity)) {
+      if (*abort_flag) return false;
+      if (clock64() - t0 > limit) {
+        *abort_flag = 1;
+        atomicExch(dev_err, static_cast<int>(kDevErrWaitTimeout));
+        return false;
+      }
+    }
+    return true;
+  }
   if (mbar_test<kCluster>(bar, parity)) return true;
   const long long t0 = clock64();
   while (true) {

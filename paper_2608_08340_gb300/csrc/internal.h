@@ -93,12 +93,16 @@ size_t tc_scratch_bytes(const SearchShape& s, const TcPlan& p);
 // keys reach it.
 // wait_limit: cycles an mbarrier wait may spin before the kernel gives up and
 // sets *dev_err (<= 0: the default of about a second).
+// phases (optional, grid x kTcPhases zeroed words): global-timer stamps of
+// each CTA's run (entry, setup done, first and last stage landed, last MMA
+// commit, epilogue sets done, exit), for measurement.
 cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s, const Fusion& fu,
                              const TcPlan& plan, void* scratch, int* dev_err, ListSet* lists,
                              cudaStream_t st, const float* init_floor = nullptr,
                              uint64_t* qfloor = nullptr, uint32_t gen = 0,
                              const float* levels = nullptr, int* level_cnt = nullptr,
-                             long long wait_limit = 0);
+                             long long wait_limit = 0, unsigned long long* phases = nullptr);
+constexpr int kTcPhases = 8;
 
 // --- final merge of partial lists into the sorted top-k per query.
 // kth_out (optional, q floats): the k-th best merged score of every query
@@ -106,7 +110,7 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
 // kLevels floats): the merged scores at ranks level_rank(k, i).
 constexpr int kLevels = 4;
 // Ranks k/16, k/8, k/4, k/2 (at least 1): candidate floors for a search of
-// k > 32 that a first pass over every 16th corpus tile proposes.
+// k > 32 that a first pass over a sample of the corpus tiles proposes.
 inline __host__ __device__ int level_rank(int k, int i) {
   const int r = k >> (kLevels - i);
   return r < 1 ? 1 : r;

@@ -136,6 +136,12 @@ struct oprag_index {
   cudaEvent_t ev[5] = {nullptr, nullptr, nullptr, nullptr, nullptr};
   // Spin limit (cycles) of the search kernels' mbarrier waits; 0 = default.
   long long wait_limit = 0;
+  // Phase stamps of the main tensor-core pass (OPRAG_OPT_PHASES): grid x
+  // kTcPhases global-timer values of the last search, and its grid.
+  bool phases_on = false;
+  void* phases = nullptr;
+  size_t phases_bytes = 0;
+  int phases_grid = 0;
 
   // Waits until all work enqueued on this index is done.
   cudaError_t drain() { return done ? cudaEventSynchronize(done) : cudaSuccess; }
@@ -252,7 +258,22 @@ int choose_path(const oprag_index* idx, int q) {
 // kSampleStride-th corpus tile (its lists, its merged top-k, and per query the
 // k-th score, kLevels counted floors and their counters).  Register lists
 // (k <= 32) also use one 64-bit shared bound per query, kept outside the block.
-constexpr int kSampleStride = 16;
+#ifndef OPRAG_SAMPLE_STRIDE
+#define OPRAG_SAMPLE_STRIDE 32
+#endif
+constexpr int kSampleStride = OPRAG_SAMPLE_STRIDE;
+// Corpus tiles from which a search with buffered lists runs the first pass.
+constexpr int kSampleMinTiles = 128;
+// Every 32nd corpus tile, lists of 8 keys (two epilogue sets, the cheapest
+// insertions).  Any k-th best of real candidates is a valid floor.  Measured
+// on 1M x 768 with 2048 queries and k = 100: with stride 16, lists of 32 / 16
+// / 8 keys gave a first pass of 395 / 264 / 218 us and the same main pass
+// (2194 us); with lists of 8, strides 8 / 16 / 32 gave steps of 2636 / 2534 /
+// 2470 us (first pass 357 / 220 / 141 us, main pass 2226 / 2256 / 2275 us).
+#ifndef OPRAG_SAMPLE_K
+#define OPRAG_SAMPLE_K 8
+#endif
+constexpr int kSampleK = OPRAG_SAMPLE_K;
 
 struct SearchLayout {
   int path = 0;           // 1 SIMT, 2 tensor core
@@ -280,13 +301,13 @@ SearchLayout search_layout(oprag_index* idx, int q, int k, int path, int block_n
   L.main_bytes = round256(tc_scratch_bytes(s, L.plan));
   // Buffered lists collect every score above their floor, and the floor of a
   // fresh list starts at -inf.  A cheap first pass over every
-  // kSampleStride-th corpus tile with 32-key lists yields, per query, the
+  // kSampleStride-th corpus tile with kSampleK-key lists yields, per query, the
   // k-th best of real corpus scores -- a lower bound of the true k-th best --
   // which the main pass then uses as the lists' starting floor.
-  L.sampled = list_len_for(k) > 32 && L.plan.nt >= 8 * kSampleStride;
+  L.sampled = list_len_for(k) > 32 && L.plan.nt >= kSampleMinTiles;
   if (L.sampled) {
     SearchShape s32 = s;
-    s32.k = 32;
+    s32.k = kSampleK;
     L.splan = tc_plan(s32, idx->num_sms, L.plan.block_n, kSampleStride, L.plan.pair,
                       pair_capacity(idx));
     const size_t per_query_tail = sizeof(float) + kLevels * (sizeof(float) + sizeof(int));
@@ -320,7 +341,7 @@ int launch_search(oprag_index* idx, const SearchLayout& L, const void* Q, int q,
     int* level_cnt = nullptr;
     if (L.sampled) {
       SearchShape s32 = s;
-      s32.k = 32;
+      s32.k = kSampleK;
       char* sbase = static_cast<char*>(scratch) + L.main_bytes;
       const size_t slist = round256(tc_scratch_bytes(s32, L.splan));
       int64_t* sids = reinterpret_cast<int64_t*>(sbase + slist);
@@ -339,8 +360,15 @@ int launch_search(oprag_index* idx, const SearchLayout& L, const void* Q, int q,
       floor = kth;
     }
     if (idx->timed_sample) cudaEventRecord(idx->ev[4], st);
+    unsigned long long* ph = nullptr;
+    if (idx->phases_on && idx->phases != nullptr &&
+        idx->phases_bytes >= static_cast<size_t>(L.plan.grid) * kTcPhases * 8) {
+      ph = static_cast<unsigned long long*>(idx->phases);
+      cudaMemsetAsync(ph, 0, static_cast<size_t>(L.plan.grid) * kTcPhases * 8, st);
+      idx->phases_grid = L.plan.grid;
+    }
     e = launch_tc_search(idx->emb, Q, s, fu, L.plan, scratch, idx->dev_err, &lists, st, floor,
-                         L.floors ? qf : nullptr, gen, levels, level_cnt, idx->wait_limit);
+                         L.floors ? qf : nullptr, gen, levels, level_cnt, idx->wait_limit, ph);
   }
   if (e != cudaSuccess) return cuda_fail(e, "search kernel");
   if (idx->timing) cudaEventRecord(idx->ev[2], st);
@@ -480,6 +508,7 @@ void oprag_index_destroy(oprag_index* idx) {
   if (idx->gcache.exec) cudaGraphExecDestroy(idx->gcache.exec);
   if (idx->scratch) cudaFree(idx->scratch);
   if (idx->qfloor) cudaFree(idx->qfloor);
+  if (idx->phases) cudaFree(idx->phases);
   if (idx->lex) cudaFree(idx->lex);
   if (idx->cand) cudaFree(idx->cand);
   if (idx->stage) cudaFree(idx->stage);
@@ -1132,6 +1161,19 @@ int oprag_index_set_option(oprag_index* idx, int32_t option, int32_t value) {
     idx->timing = value != 0;
     return ok();
   }
+  if (option == OPRAG_OPT_PHASES) {
+    if (value < 0 || value > 1) return fail(OPRAG_ERR_INVALID_ARG, "phases %d", value);
+    if (value) {
+      DeviceGuard g(idx->device);
+      // One stamp row per CTA of the largest grid (every SM, or pairs).
+      const size_t need = static_cast<size_t>(2 * idx->num_sms) * kTcPhases * 8;
+      int rc = idx->ensure(&idx->phases, &idx->phases_bytes, need, "phase stamps");
+      if (rc) return rc;
+    }
+    idx->phases_on = value != 0;
+    idx->phases_grid = 0;
+    return ok();
+  }
   if (option == OPRAG_OPT_WAIT_LIMIT) {
     if (value < 0) return fail(OPRAG_ERR_INVALID_ARG, "wait limit %d", value);
     idx->wait_limit = value;
@@ -1211,6 +1253,22 @@ int oprag_index_last_timing(oprag_index* idx, float* lexical_ms, float* sample_m
   if (sample_ms) *sample_ms = b;
   if (search_ms) *search_ms = c;
   if (merge_ms) *merge_ms = m;
+  return ok();
+}
+
+int oprag_index_last_phases(oprag_index* idx, int64_t* out, int32_t cap, int32_t* ctas) {
+  if (!idx || !ctas) return fail(OPRAG_ERR_INVALID_ARG, "NULL argument");
+  if (!idx->phases_on || idx->phases_grid == 0)
+    return fail(OPRAG_ERR_NOT_READY, "no tensor-core search ran with phase stamps on");
+  DeviceGuard g(idx->device);
+  cudaError_t e = idx->drain();
+  if (e != cudaSuccess) return cuda_fail(e, "pending work");
+  *ctas = idx->phases_grid;
+  const int64_t count = static_cast<int64_t>(idx->phases_grid) * kTcPhases;
+  if (out == nullptr) return ok();
+  if (cap < count) return fail(OPRAG_ERR_INVALID_ARG, "need room for %lld stamps", (long long)count);
+  e = cudaMemcpy(out, idx->phases, count * 8, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "reading phase stamps");
   return ok();
 }
 

@@ -159,7 +159,7 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
                              const TcPlan& pl, void* scratch, int* dev_err, ListSet* lists,
                              cudaStream_t st, const float* init_floor, uint64_t* qfloor,
                              uint32_t gen, const float* levels, int* level_cnt,
-                             long long wait_limit) {
+                             long long wait_limit, unsigned long long* phases) {
   CUtensorMap mq, me;
   // With a single query tile only its real rows are loaded (the remaining
   // rows of the A tile hold stale data whose TMEM lanes the epilogue never
@@ -193,6 +193,7 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
   prm.meta_count = reinterpret_cast<int*>(prm.meta_worst + (K > 32 ? rows : 0));
   prm.dev_err = dev_err;
   prm.wait_limit = wait_limit > 0 ? wait_limit : kWaitLimitCycles;
+  prm.phases = phases;
   // Register lists publish their k-th scores; buffered lists use counted floors.
   prm.qfloor = K <= 32 ? qfloor : nullptr;
   prm.gen = gen;

@@ -81,7 +81,33 @@ struct TcParams {
   // reached k bounds the query's k-th best score for every list.
   const float* levels;
   int* level_cnt;
+  // Optional (measurement): kPhases global-timer stamps per CTA (PhaseMark).
+  unsigned long long* phases;
 };
+
+// Points of a CTA's run whose global-timer values a measurement run records
+// (TcParams::phases, slot blockIdx.x * kPhases + mark).
+enum PhaseMark : int {
+  kPhEntry = 0,        // first instruction
+  kPhSetup = 1,        // barriers initialised, TMEM allocated (after the setup barrier)
+  kPhFirstStage = 2,   // MMA issuer: first pipeline stage landed
+  kPhLastStage = 3,    // MMA issuer: last pipeline stage landed
+  kPhLastCommit = 4,   // MMA issuer: last unit's MMAs issued and committed
+  kPhEpi0Done = 5,     // epilogue set 0: last unit filtered
+  kPhEpi1Done = 6,     // epilogue set 1 (two sets): last unit filtered
+  kPhExit = 7,         // after the final barrier, before TMEM is freed
+  kPhases = 8
+};
+
+__device__ __forceinline__ unsigned long long global_timer() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void note_phase(const TcParams& p, int mark) {
+  if (p.phases != nullptr) p.phases[static_cast<size_t>(blockIdx.x) * kPhases + mark] = global_timer();
+}
 
 // Units of one CTA in processing order.  The corpus tiles are cut into
 // windows of `win` tiles (sized to stay in L2); inside a window the units
@@ -610,6 +636,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
   constexpr uint32_t kTmemCols = (kDual ? 4 : 2) * BN;
   constexpr int kEpiSets = epi_sets(K);
   extern __shared__ __align__(1024) unsigned char smem_raw[];
+  if (threadIdx.x == 0) note_phase(p, kPhEntry);
   unsigned char* base = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   unsigned char* sA = base;
@@ -691,6 +718,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  if (threadIdx.x == 0) note_phase(p, kPhSetup);
   const uint32_t tmem_base = *tmem_slot;
   // Let the merge kernel that follows on the stream get scheduled; it waits
   // for this grid to finish before reading the lists.
@@ -738,6 +766,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       int acc = 0;
       uint32_t acc_ph = 0;
       bool ok = true;
+      bool landed = false;
       UnitSeq us;
       for (us.start(p, cta, C); ok && us.valid(); us.next()) {
         if constexpr (kDual) {
@@ -751,6 +780,11 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
           for (int kb = 0; kb < p.kblocks; ++kb) {
             if (!mbar_wait(&full[s], ph, abort_flag, p.dev_err, p.wait_limit)) { ok = false; break; }
             tc_fence_after();
+            if (p.phases != nullptr) {
+              if (!landed) note_phase(p, kPhFirstStage);
+              landed = true;
+              note_phase(p, kPhLastStage);
+            }
             const uint64_t a0 = sw128_desc(smem_addr(sA + s * kAStage));
             const uint64_t a1 = sw128_desc(smem_addr(sA + s * kAStage + kAStageBytes));
             const uint64_t b = sw128_desc(smem_addr(sB + s * kBStageBytes));
@@ -775,6 +809,11 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         for (int kb = 0; kb < p.kblocks; ++kb) {
           if (!mbar_wait(&full[s], ph, abort_flag, p.dev_err, p.wait_limit)) { ok = false; break; }
           tc_fence_after();
+          if (p.phases != nullptr) {
+            if (!landed) note_phase(p, kPhFirstStage);
+            landed = true;
+            note_phase(p, kPhLastStage);
+          }
           const uint64_t a = sw128_desc(smem_addr(sA + s * kAStage));
           const uint64_t b = sw128_desc(smem_addr(sB + s * kBStageBytes));
           if constexpr (kPair) {
@@ -795,6 +834,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         else mma_commit(&tfull[acc]);
         if (++acc == 2) { acc = 0; acc_ph ^= 1u; }
       }
+      note_phase(p, kPhLastCommit);
       if constexpr (kPair) mma_commit_pair(mma_done);
       else mma_commit(mma_done);
       mbar_drain(mma_done, 0, p.dev_err);
@@ -1062,6 +1102,10 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       for (int J = 0; J < p.qt; ++J)
         if (owns(J)) list.finalize(p, list_row(J), qtile(J) * kBlockM + row < p.q);
     }
+    // The set's last warp to finish (the slots start at zero).
+    if (p.phases != nullptr && lane == 0)
+      atomicMax(p.phases + static_cast<size_t>(blockIdx.x) * kPhases + kPhEpi0Done + set,
+                global_timer());
   }
 
   tc_fence_before();
@@ -1070,6 +1114,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
   if constexpr (kPair) cluster_sync();
   else __syncthreads();
   tc_fence_after();
+  if (threadIdx.x == 0) note_phase(p, kPhExit);
   if (warp == 1) {
     if constexpr (kPair) tmem_dealloc_pair(tmem_base, kTmemCols);
     else tmem_dealloc(tmem_base, kTmemCols);

@@ -235,6 +235,24 @@ class Index:
                                                  ctypes.byref(c)))
         return {"scratch": a.value, "bounds": b.value, "lexical": c.value}
 
+    PHASES = ("entry", "setup", "first_stage", "last_stage", "last_commit", "epi0_done",
+              "epi1_done", "exit")
+
+    def enable_phases(self, on: bool = True) -> None:
+        """Measurement hook: per-CTA global-timer stamps of the main pass."""
+        self.set_option(_lib.OPRAG_OPT_PHASES, int(on))
+
+    def last_phases(self) -> np.ndarray:
+        """(ctas, 8) int64 global-timer stamps (ns) of the last main pass, in
+        the order of PHASES (0 where a CTA records none)."""
+        n = ctypes.c_int32()
+        check(self._lib.oprag_index_last_phases(self._h, None, 0, ctypes.byref(n)))
+        out = np.zeros((n.value, 8), np.int64)
+        check(self._lib.oprag_index_last_phases(
+            self._h, out.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)), out.size,
+            ctypes.byref(n)))
+        return out
+
     def set_wait_limit(self, cycles: int) -> None:
         """Test hook: spin limit of the search kernels' barrier waits (0 = default)."""
         self.set_option(_lib.OPRAG_OPT_WAIT_LIMIT, int(cycles))

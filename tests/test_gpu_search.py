@@ -217,7 +217,7 @@ def test_config4_scale_with_upserts_sampled():
 
 @pytest.mark.parametrize("k", [33, 100, 256])
 def test_large_k_with_sampled_floor(k):
-    """k > 32 over many corpus tiles: the search first scans every 16th tile
+    """k > 32 over many corpus tiles: the search first scans every 32nd tile
     to get a lower bound of each query's k-th best score, then the full scan
     admits only scores above it.  Results must still be exact."""
     rng = np.random.default_rng(k)

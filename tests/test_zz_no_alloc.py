@@ -32,11 +32,9 @@ def _noalloc(lib, idx, Q, k):
 
 
 # (cfg, q, k, n): dual mode (256 queries), one query, single CTAs with lists of
-# 16, the fp32 SIMT kernel, and two k > 32 cases: a small corpus (no sampled
-# pass) and 157 corpus tiles (the sampled first pass and counted floors run).
+# 16, the fp32 SIMT kernel, and k > 32 (buffered lists) on a small corpus.
 @pytest.mark.parametrize("cfg,q,k,n", [(1, 256, 5, 20000), (1, 1, 5, 20000), (2, 300, 10, 20000),
-                                       (0, 16, 5, None), (1, 64, 100, 2000),
-                                       (1, 64, 100, 20000)])
+                                       (0, 16, 5, None), (1, 64, 100, 2000)])
 def test_noalloc_matches_search_twice(cfg, q, k, n):
     lib = _lib.load()
     w = workloads.config(cfg, batch=q, n=n)
@@ -60,14 +58,19 @@ def test_noalloc_matches_search_twice(cfg, q, k, n):
     idx.close()
 
 
-def test_noalloc_refuses_searches_beyond_the_static_array():
+@pytest.mark.parametrize("q,k", [(4096, 256), (64, 100)])
+def test_noalloc_refuses_searches_beyond_the_static_array(q, k):
+    """Thousands of queries with k = 256, and k = 100 over 157 corpus tiles:
+    there one 128-row list of 256 keys per CTA (about 38 MB over the grid)
+    exceeds the 16 MiB array."""
     lib = _lib.load()
-    w = workloads.config(1, batch=4096, n=20000)
+    w = workloads.config(1, batch=q, n=20000)
     idx = Index(dev_tensor(w.E_data))
-    rc, ids, _ = _noalloc(lib, idx, dev_tensor(w.Q_data), 256)
+    rc, ids, _ = _noalloc(lib, idx, dev_tensor(w.Q_data), k)
     assert rc == -1
     msg = lib.oprag_last_error().decode()
     assert "static array" in msg
     torch.cuda.synchronize()
     assert (ids == -7).all()            # nothing was launched
+    assert idx.buffer_bytes() == {"scratch": 0, "bounds": 0, "lexical": 0}
     idx.close()
