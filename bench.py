@@ -108,6 +108,9 @@ def parse(argv=None):
     p.add_argument("--index-ops", action="store_true",
                    help="time the index updates instead: append of 4096 rows, replacement of "
                         "4096 token bags (BM25 rebuilt), search over a knowledge + memory index")
+    p.add_argument("--lex-gather", action="store_true",
+                   help="config 3: gather BM25 in the search epilogue (OPRAG_OPT_LEX_GATHER) "
+                        "instead of reading a materialised BM25 block")
     p.add_argument("--dense-first", type=int, default=0, metavar="N",
                    help="config 3 only: dense top-N, then the lexical rerank of those N "
                         "candidates (dense-first hybrid) instead of the full hybrid")
@@ -383,6 +386,7 @@ def measure(args, cfg: int, batch: int, rank: int, world: int, local_rank: int,
     idx = Index(_to_dev(w.E_data, dev))
     if cfg == 3:
         idx.set_sparse(w.doc_indptr, w.doc_terms, w.vocab, w.k1, w.b)
+        idx.gather_lexical(bool(args.lex_gather))
         q_indptr = torch.from_numpy(w.q_indptr).to(dev)
         q_terms = torch.from_numpy(w.q_terms).to(dev)
     idx.force_block_n(args.block_n or None)
@@ -606,6 +610,10 @@ def measure(args, cfg: int, batch: int, rank: int, world: int, local_rank: int,
     if cfg == 3:
         h2d += w.q_indptr.nbytes + w.q_terms.nbytes
     d2h = w.q * w.k * 12
+    lex_form = None
+    if cfg == 3 and not dense_first:
+        lex_form = ("gathered in the search epilogue (no BM25 block)" if args.lex_gather else
+                    "materialised q x n BM25 block read by the search epilogue")
     result = {
         "metric": f"queries/s at top-{w.k}", "value": job_rate(w.q, args.steps, world, total_ms),
         "unit": "queries/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
@@ -635,6 +643,8 @@ def measure(args, cfg: int, batch: int, rank: int, world: int, local_rank: int,
         result["quality"] = quality
     if phases:
         result["phases"] = phases
+    if lex_form:
+        result["lexical"] = lex_form
     extra = {"ids": out_ids, "scores": out_scores,
              "upserts": ([(ups[r][0], ups[r][1]) for r in upsert_sequence(args.warmup, args.steps)]
                          if cfg == 4 else [])}
@@ -678,7 +688,8 @@ def phase_breakdown(idx, step, flush, n_steps: int) -> dict:
 def sub_entry(res: dict) -> dict:
     """The fields of a workload's line kept under the headline's "configs"."""
     keep = ("value", "unit", "ms_per_step", "ms_per_step_median", "roofline", "e2e", "clocks",
-            "warm_l2", "parity", "gpu_launches", "path", "launch", "upsert", "metric", "phases")
+            "warm_l2", "parity", "gpu_launches", "path", "launch", "upsert", "metric", "phases",
+            "lexical")
     out = {k: res[k] for k in keep if k in res}
     out["workload"] = res["config"]["workload"]
     return out

@@ -293,6 +293,19 @@ OPRAG_API int oprag_index_set_option(oprag_index *idx, int32_t option, int32_t v
  * the waits of a real search run out. */
 #define OPRAG_OPT_WAIT_LIMIT 7
 
+/* OPRAG_OPT_LEX_GATHER (tensor-core path): how oprag_hybrid_search gets the
+ * lexical half.  0 (default): a BM25 pass writes the q x n block of BM25
+ * values (up to 2^28 values per pass) that the search's fused selection
+ * reads.  1: nothing of that size is written -- a pass computes only each
+ * query's BM25 maximum, and the search gathers BM25(q, d) in its epilogue:
+ * the 32 commonest terms through one more tensor-core K block (the query's
+ * term counts times each chunk's weights split into a high and a low bf16
+ * half, within 2^-18 of the weight), terms in at least 1/32 of the chunks as
+ * rows of fp32 weights, the others from their postings.  Same results
+ * within the 1e-4 score bar; on 32768 x 768 with 1024 queries of 8 Zipf
+ * terms the default measured 4x faster. */
+#define OPRAG_OPT_LEX_GATHER 9
+
 /* OPRAG_OPT_PHASES (measurement hook): 1 makes the main tensor-core pass of
  * every later search record, per CTA, the GPU global timer (nanoseconds) at
  * eight points of its run; oprag_index_last_phases() reads them.  Costs one

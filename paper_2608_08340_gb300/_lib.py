@@ -20,6 +20,7 @@ OPRAG_OPT_BOUND_TAG = 5
 OPRAG_OPT_GRAPH = 6
 OPRAG_OPT_WAIT_LIMIT = 7
 OPRAG_OPT_PHASES = 8
+OPRAG_OPT_LEX_GATHER = 9
 
 ERRORS = {
     0: "OK",

@@ -132,10 +132,11 @@ bm25_matrix_kernel(SparseIndex sp, int64_t n, const int32_t* __restrict__ q_indp
   }
 
   float m = 0.f;
-  float4* orow = reinterpret_cast<float4*>(out + static_cast<int64_t>(qi) * ld + d0);
+  float4* orow =
+      out != nullptr ? reinterpret_cast<float4*>(out + static_cast<int64_t>(qi) * ld + d0) : nullptr;
   for (int i = threadIdx.x; i < nv; i += blockDim.x) {
     const float4 v = acc4[i];
-    orow[i] = v;
+    if (orow != nullptr) orow[i] = v;
     m = fmaxf(fmaxf(m, fmaxf(v.x, v.y)), fmaxf(v.z, v.w));
   }
 #pragma unroll
@@ -150,7 +151,73 @@ bm25_matrix_kernel(SparseIndex sp, int64_t n, const int32_t* __restrict__ q_indp
   }
 }
 
+// One thread per query, by the classes of its terms: the head terms' counts
+// (as bf16, twice: against the high and the low half of the split weights),
+// its first kLexMidReg distinct mid rows and first kLexRegTerms distinct tail
+// terms that have postings, each with its multiplicity, in first-occurrence
+// order, and the raw term index where a further distinct one first occurs
+// (the end of the query's terms if none does).
+__global__ void lex_prep_kernel(const int32_t* __restrict__ lex_class,
+                                const int64_t* __restrict__ post_ptr, int vocab,
+                                const int32_t* __restrict__ q_indptr,
+                                const int32_t* __restrict__ q_terms, int q, LexPrep out) {
+  const int qi = blockIdx.x * blockDim.x + threadIdx.x;
+  if (qi >= q) return;
+  float cnt[kLexHeadTerms];
+#pragma unroll
+  for (int i = 0; i < kLexHeadTerms; ++i) cnt[i] = 0.f;
+  const int t0 = q_indptr[qi], t1 = q_indptr[qi + 1];
+  int4* tails = out.terms + static_cast<int64_t>(qi) * kLexRegTerms;
+  int2* mids = out.mid + static_cast<int64_t>(qi) * kLexMidReg;
+  int nt = 0, nm = 0, first_ovf = t1;
+  for (int i = t0; i < t1; ++i) {
+    const int32_t term = q_terms[i];
+    if (term < 0 || term >= vocab) continue;
+    const int c = lex_class[term];
+    if (c >= 0) {
+#pragma unroll
+      for (int s = 0; s < kLexHeadTerms; ++s) cnt[s] += s == c ? 1.f : 0.f;
+    } else if (c <= -2) {
+      const int row = -2 - c;
+      int j = 0;
+      while (j < nm && mids[j].x != row) ++j;
+      if (j < nm) mids[j].y = __float_as_int(__int_as_float(mids[j].y) + 1.f);
+      else if (nm < kLexMidReg) mids[nm++] = make_int2(row, __float_as_int(1.f));
+      else if (first_ovf == t1) first_ovf = i;
+    } else {
+      const int64_t a = post_ptr[term], b = post_ptr[term + 1];
+      if (a >= b) continue;
+      int j = 0;
+      while (j < nt && tails[j].w != term) ++j;
+      if (j < nt)
+        tails[j].z = __float_as_int(__int_as_float(tails[j].z) + 1.f);
+      else if (nt < kLexRegTerms)
+        tails[nt++] = make_int4(static_cast<int>(a), static_cast<int>(b), __float_as_int(1.f), term);
+      else if (first_ovf == t1)
+        first_ovf = i;
+    }
+  }
+  out.term_cnt[qi] = nt;
+  out.mid_cnt[qi] = nm;
+  out.ovf[qi] = first_ovf;
+  __nv_bfloat16* row = static_cast<__nv_bfloat16*>(out.qcount) + static_cast<int64_t>(qi) * kLexK;
+#pragma unroll
+  for (int s = 0; s < kLexHeadTerms; ++s) {
+    row[s] = __float2bfloat16_rn(cnt[s]);
+    row[kLexHeadTerms + s] = __float2bfloat16_rn(cnt[s]);
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_lex_prep(const int32_t* lex_class, const int64_t* post_ptr, int vocab,
+                            const int32_t* q_indptr, const int32_t* q_terms, int q,
+                            const LexPrep& out, cudaStream_t st) {
+  if (q <= 0) return cudaSuccess;
+  lex_prep_kernel<<<(q + 127) / 128, 128, 0, st>>>(lex_class, post_ptr, vocab, q_indptr, q_terms,
+                                                   q, out);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_bm25_matrix(const SparseIndex& sp, int64_t n, const int32_t* q_indptr,
                                const int32_t* q_terms, int q, float* out, int64_t ld,

@@ -36,13 +36,50 @@ struct ListSet {
 };
 
 // Optional lexical part of the fused score (Sec. 4.4 weighted fusion):
-// f = alpha * dense + (1 - alpha) * bm25[q][id] / max_q, zero lexical part when
-// max_q <= 0.  bm25 == nullptr means a plain dense search.
+// f = alpha * dense + (1 - alpha) * BM25(q, id) / max_q, zero lexical part when
+// max_q <= 0.  Two forms:
+//  * materialised (SIMT kernel): bm25 is a q x ld block of BM25 values;
+//  * gathered in the tensor-core epilogue (bm25 == nullptr, lex_qcount set).
+//    Each term of the sparse side has a class (lex_class):
+//    - head (class s in [0, kLexHeadTerms)): one more K block of tensor-core
+//      MMAs, lex_qcount (q x kLexK bf16: the query's count of each head
+//      term, twice) times lex_wsplit (n x kLexK bf16: each chunk's head-term
+//      weights split into a high and a low bf16 half), accumulated in fp32;
+//    - mid (class -2 - r): row r of mid_w (fp32 weight per chunk, mid_ld
+//      apart), read per chunk;
+//    - tail (class -1): its postings (lex_post, chunks ascending), walked per
+//      chunk with a cursor.
+//    Per query the prep kernel lists up to kLexMidReg mid rows (lex_mid: row,
+//    multiplicity bits) and kLexRegTerms tail terms (lex_terms: first
+//    posting, end posting, multiplicity bits, term id); further terms of a
+//    long query are handled by scanning its raw terms from lex_ovf[q] on.
+// Neither (bm25 == nullptr and lex_qcount == nullptr) means a plain dense search.
+constexpr int kLexHeadTerms = 32;              // head terms scored on tensor cores
+constexpr int kLexK = 2 * kLexHeadTerms;       // one 64-element K block: high | low halves
+constexpr int kLexRegTerms = 8;                // tail terms with a cursor per thread
+constexpr int kLexMidReg = 2;                  // mid rows per query read with cp.async
 struct Fusion {
   const float* bm25;      // q x ld, row-major
   int64_t ld;
   const float* bm25_max;  // q
   float alpha;
+  const void* lex_qcount = nullptr;
+  const void* lex_wsplit = nullptr;
+  const int4* lex_terms = nullptr;    // q x kLexRegTerms
+  const int* lex_term_cnt = nullptr;  // q
+  const int2* lex_mid = nullptr;      // q x kLexMidReg
+  const int* lex_mid_cnt = nullptr;   // q
+  const int* lex_ovf = nullptr;       // q
+  const int2* lex_post = nullptr;
+  const float* mid_w = nullptr;
+  int64_t mid_ld = 0;                 // multiple of 128, >= n
+  // for the scan of long queries: the query CSR and the term tables
+  const int32_t* q_indptr = nullptr;
+  const int32_t* q_terms = nullptr;
+  const int32_t* lex_class = nullptr;
+  const int64_t* post_ptr = nullptr;
+  int vocab = 0;
+  bool gathered() const { return lex_qcount != nullptr; }
 };
 
 struct SearchShape {
@@ -50,6 +87,9 @@ struct SearchShape {
   int d;
   int q;
   int k;
+  // The lexical part is gathered in the tensor-core epilogue: the plan uses
+  // single CTAs with 128-row corpus tiles and one epilogue set.
+  bool fused_lex = false;
 };
 
 // --- SIMT streaming search (fp32 or bf16; any q, meant for small q).
@@ -147,9 +187,25 @@ struct SparseIndex {
   const int64_t* tile_ptr;
   int ntiles;
 };
+// out == nullptr computes only the per-query maxima (the gathered form).
 cudaError_t launch_bm25_matrix(const SparseIndex& sp, int64_t n, const int32_t* q_indptr,
                                const int32_t* q_terms, int q, float* out, int64_t ld,
                                float* out_max, cudaStream_t st);
+
+// Per-query operands of the gathered lexical part (see Fusion): qcount
+// (q x kLexK bf16), terms (q x kLexRegTerms), mid (q x kLexMidReg) and the
+// counts term_cnt, mid_cnt and ovf (q each), from the terms' classes.
+struct LexPrep {
+  void* qcount;
+  int4* terms;
+  int* term_cnt;
+  int2* mid;
+  int* mid_cnt;
+  int* ovf;
+};
+cudaError_t launch_lex_prep(const int32_t* lex_class, const int64_t* post_ptr, int vocab,
+                            const int32_t* q_indptr, const int32_t* q_terms, int q,
+                            const LexPrep& out, cudaStream_t st);
 
 // --- lexical rerank of a dense top-N (dense-first hybrid), rerank.cu.
 // cand_ids / cand_scores: q x ncand dense results (id -1 = none), ncand <=

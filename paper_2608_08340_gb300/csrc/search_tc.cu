@@ -56,7 +56,11 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
   TcPlan pl{};
   pl.qt = (s.q + kBlockM - 1) / kBlockM;
   int bn = 256;
-  if (force_block_n == 128 || force_block_n == 256) {
+  if (s.fused_lex) {
+    // The gathered hybrid search: single CTAs, 128-row tiles, one epilogue
+    // set (its accumulators take all 512 TMEM columns).
+    bn = 128;
+  } else if (force_block_n == 128 || force_block_n == 256) {
     bn = force_block_n;
   } else {
     // Few units (small query batches): 128-row tiles give every SM more of
@@ -71,8 +75,8 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
   // CTA (small batches, where the copies into the SMs, not the MMAs, bound
   // the kernel; measured on 32768 x 768: faster up to 512 queries, slower at
   // 1024); it needs the two epilogue sets of lists of 8 or 16.
-  const bool dual_ok = pl.qt >= 2 && epi_sets(list_len_for(s.k)) == 2 && force_pair != 2 &&
-                       (force_block_n == 0 || force_block_n == 128);
+  const bool dual_ok = !s.fused_lex && pl.qt >= 2 && epi_sets(list_len_for(s.k)) == 2 &&
+                       force_pair != 2 && (force_block_n == 0 || force_block_n == 128);
   const int64_t dual_units = static_cast<int64_t>((pl.qt + 1) / 2) * ((s.n + 127) / 128);
   pl.dual = dual_ok && (force_pair == 3 || (force_pair == 0 && dual_units <= 4LL * num_sms));
   if (pl.dual) bn = 128;
@@ -83,7 +87,7 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
   // (k > 32, at least 8 query tiles): measured on GB300, 1M x 768 with 2048
   // queries and k = 100 takes 2524 instead of 2591 us; with lists of 16
   // (32768 x 1024, 4096 queries, k = 10) pairs are no faster.
-  const bool pair = bn == 256 && pair_capacity > 0 &&
+  const bool pair = !s.fused_lex && bn == 256 && pair_capacity > 0 &&
                     (force_pair == 2 ||
                      (force_pair == 0 && list_len_for(s.k) > 32 && pl.qt >= 8));
   pl.pair = pair ? 2 : 1;
@@ -127,16 +131,18 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
   for (int j = 0; j < pl.uqt; ++j)
     per_tile = std::max(per_tile, hi[j] - first_cta(j, pl.uqt, C) + 1);
   if (!ok) per_tile = C;  // not expected; every slot then gets a list per tile
-  pl.pmax = per_tile * (pl.dual ? 1 : epi_sets(list_len_for(s.k)));
+  pl.pmax = per_tile * (pl.dual ? 1 : epi_sets(list_len_for(s.k), s.fused_lex));
   const int K = list_len_for(s.k);
   // Shared memory of the launch (the same sum as smem_for<BN, K, pair, dual>).
   const size_t b_stage = static_cast<size_t>(pair ? bn / 2 : bn) * 128;
   const size_t a_stage = kAStageBytes * (pl.dual ? 2 : 1);
-  pl.stages = pair      ? stages_for<256, true>()
-              : pl.dual ? stages_for<128, false, true>()
-                        : (bn == 128 ? stages_for<128>() : stages_for<256>());
+  pl.stages = pair        ? stages_for<256, true>()
+              : pl.dual     ? stages_for<128, false, true>()
+              : s.fused_lex ? stages_for<128, false, false, true>()
+                            : (bn == 128 ? stages_for<128>() : stages_for<256>());
   pl.smem = static_cast<size_t>(pl.stages) * (a_stage + b_stage) +
-            static_cast<size_t>(epi_sets(K)) * 128 * kStageRowBytes + 1024 + 256;
+            static_cast<size_t>(epi_sets(K, s.fused_lex)) * 128 * kStageRowBytes +
+            lex_land_bytes(s.fused_lex) + 1024 + 256;
   return pl;
 }
 
@@ -160,7 +166,7 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
                              cudaStream_t st, const float* init_floor, uint64_t* qfloor,
                              uint32_t gen, const float* levels, int* level_cnt,
                              long long wait_limit, unsigned long long* phases) {
-  CUtensorMap mq, me;
+  TcMaps maps;
   // With a single query tile only its real rows are loaded (the remaining
   // rows of the A tile hold stale data whose TMEM lanes the epilogue never
   // reads); rows are loaded in multiples of 8, the swizzle atom height.
@@ -168,9 +174,22 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
   // corpus tile.
   const int a_rows =
       pl.qt == 1 && pl.pair == 1 && !pl.dual ? std::min(kBlockM, (s.q + 7) / 8 * 8) : kBlockM;
-  if (!make_map(&mq, Q, s.q, s.d, a_rows) ||
-      !make_map(&me, E, s.n, s.d, pl.block_n / pl.pair))
+  if (!make_map(&maps.q, Q, s.q, s.d, a_rows) ||
+      !make_map(&maps.e, E, s.n, s.d, pl.block_n / pl.pair))
     return cudaErrorInvalidValue;
+  const bool hybrid = fu.gathered();
+  const int lex = hybrid ? kLexGather : fu.bm25 != nullptr ? kLexBlock : kLexNone;
+  if (hybrid != s.fused_lex) return cudaErrorInvalidValue;
+  if (hybrid) {
+    // head-term counts (q x kLexK) and split weights (n x kLexK): one K block
+    if (pl.block_n != 128 || pl.pair != 1 || pl.dual ||
+        !make_map(&maps.qb, fu.lex_qcount, s.q, kLexK, a_rows) ||
+        !make_map(&maps.eb, fu.lex_wsplit, s.n, kLexK, pl.block_n))
+      return cudaErrorInvalidValue;
+  } else {
+    maps.qb = maps.q;
+    maps.eb = maps.e;
+  }
   const int K = list_len_for(s.k);
   const int stride = K > 32 ? 2 * K : K;
   const size_t rows = list_rows(pl);
@@ -205,22 +224,22 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
   lists->stride = stride;
   lists->C = pl.grid / pl.pair;
   lists->qt = pl.uqt;
-  lists->sets = pl.dual ? 1 : epi_sets(K);
+  lists->sets = pl.dual ? 1 : epi_sets(K, hybrid);
   lists->klen = K;
   lists->pair = pl.dual ? 2 : pl.pair;
-  const bool hybrid = fu.bm25 != nullptr;
+  if (hybrid) return launch_bn128_gather(maps, prm, pl.grid, st);
   if (pl.dual) {
     if (pl.block_n != 128) return cudaErrorInvalidValue;
-    return launch_dual128(mq, me, prm, pl.grid, hybrid, st);
+    return launch_dual128(maps, prm, pl.grid, lex, st);
   }
   if (pl.pair == 2) {
     if (pl.block_n != 256) return cudaErrorInvalidValue;
-    return hybrid ? launch_pair256_fused(mq, me, prm, pl.grid, st)
-                  : launch_pair256_dense(mq, me, prm, pl.grid, st);
+    return lex == kLexBlock ? launch_pair256_block(maps, prm, pl.grid, st)
+                            : launch_pair256_dense(maps, prm, pl.grid, st);
   }
-  if (pl.block_n == 128) return launch_bn128(mq, me, prm, pl.grid, hybrid, st);
-  return hybrid ? launch_bn256_fused(mq, me, prm, pl.grid, st)
-                : launch_bn256_dense(mq, me, prm, pl.grid, st);
+  if (pl.block_n == 128) return launch_bn128(maps, prm, pl.grid, lex, st);
+  return lex == kLexBlock ? launch_bn256_block(maps, prm, pl.grid, st)
+                          : launch_bn256_dense(maps, prm, pl.grid, st);
 }
 
 }  // namespace oprag

@@ -45,8 +45,14 @@ constexpr int kUmmaK = 16;
 // put three on two of the SM's four schedulers, which caps a thread at 168
 // registers; with six warps it may use 255 (measured: buffered lists with two
 // sets spill and run 11% slower).
-__host__ __device__ constexpr int epi_sets(int K) { return K <= 16 ? 2 : 1; }
-__host__ __device__ constexpr int threads_for(int K) { return 64 + 128 * epi_sets(K); }
+// The gathered hybrid search keeps one set (its postings cursors advance
+// through consecutive units).
+__host__ __device__ constexpr int epi_sets(int K, bool lex = false) {
+  return K <= 16 && !lex ? 2 : 1;
+}
+__host__ __device__ constexpr int threads_for(int K, bool lex = false) {
+  return 64 + 128 * epi_sets(K, lex);
+}
 constexpr uint32_t kAStageBytes = kBlockM * kBlockK * 2;
 constexpr int kSmemBudget = 200 * 1024;
 
@@ -173,22 +179,32 @@ constexpr uint32_t a_stage_bytes() {
   return kAStageBytes * (kDual ? 2u : 1u);
 }
 
-template <int BN, bool kPair = false, bool kDual = false>
+// Per-thread landing zone of the gathered hybrid search's copies: kLexMidReg
+// rows of 32 floats, then 2 postings per tail term; the 400-byte stride (100
+// words) spreads the lanes over the banks.  One set of 128 threads.
+constexpr int kLexLandStride = 400;
+__host__ __device__ constexpr int lex_land_bytes(bool lex) {
+  return lex ? 128 * kLexLandStride : 0;
+}
+
+template <int BN, bool kPair = false, bool kDual = false, bool kLex = false>
 constexpr int stages_for() {
-  return kSmemBudget / (a_stage_bytes<kDual>() + b_stage_bytes<BN, kPair>()) > 8
+  return (kSmemBudget - lex_land_bytes(kLex)) / (a_stage_bytes<kDual>() + b_stage_bytes<BN, kPair>()) > 8
              ? 8
-             : kSmemBudget / (a_stage_bytes<kDual>() + b_stage_bytes<BN, kPair>());
+             : (kSmemBudget - lex_land_bytes(kLex)) /
+                   (a_stage_bytes<kDual>() + b_stage_bytes<BN, kPair>());
 }
 
 // Per epilogue thread: one 32-float row where a chunk's scores are staged so
 // that candidate columns can be read back by index.
 constexpr int kStageRowBytes = 32 * 4;
 
-template <int BN, int K, bool kPair = false, bool kDual = false>
+template <int BN, int K, bool kPair = false, bool kDual = false, bool kLex = false>
 constexpr size_t smem_for() {
-  return static_cast<size_t>(stages_for<BN, kPair, kDual>()) *
+  return static_cast<size_t>(stages_for<BN, kPair, kDual, kLex>()) *
              (a_stage_bytes<kDual>() + b_stage_bytes<BN, kPair>()) +
-         static_cast<size_t>(epi_sets(K)) * 128 * kStageRowBytes + 1024 + 256;
+         static_cast<size_t>(epi_sets(K, kLex)) * 128 * kStageRowBytes + lex_land_bytes(kLex) +
+         1024 + 256;
 }
 
 // ----------------------------------------------------------------- PTX
@@ -606,6 +622,204 @@ struct EpiList<K, true> {
   }
 };
 
+// ----------------------------------------------------------- lexical gather
+// The mid and tail terms of one thread's query in the gathered hybrid search
+// (Sec. 4.4, inverted-postings BM25; see Fusion).  Per chunk of 32 corpus
+// rows the thread copies, with cp.async into its landing zone in shared
+// memory (no registers held while the copies fly), the chunk's 32 weights of
+// each listed mid row and the next two postings of each listed tail term.
+// A tail term's cursor (chunk ids ascending) is kept across the chunks and
+// units that the thread filters in increasing chunk order, so each posting
+// is read once; it is re-placed by binary search when the thread's query
+// changes or its units are not consecutive.  Tail terms have under one
+// posting per 32 chunks on average; a longer run falls back to dependent
+// loads.  Terms past the listed ones (long queries) are searched per chunk.
+
+static_assert(kLexMidReg * 128 + kLexRegTerms * 16 <= kLexLandStride, "landing zone");
+
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_addr(dst)), "l"(src)
+               : "memory");
+}
+
+__device__ __forceinline__ void cp_async8(void* dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(smem_addr(dst)), "l"(src)
+               : "memory");
+}
+
+__device__ __forceinline__ void cp_async_commit_wait_all() {
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+}
+
+struct LexCursor {
+  int base[kLexRegTerms], cur[kLexRegTerms], end[kLexRegTerms], term[kLexRegTerms];
+  float mul[kLexRegTerms];
+  int mrow[kLexMidReg];
+  float mmul[kLexMidReg];
+  int nreg = 0, nmid = 0;      // listed tail terms and mid rows
+  int ovf = 0, ovf_end = 0;    // raw term range scanned for further terms
+  int64_t next_doc = -1;       // first chunk that continues the cursors (-1: none)
+
+  __device__ __forceinline__ void set_query(const TcParams& p, int64_t qi) {
+    nreg = p.fu.lex_term_cnt[qi];
+    nmid = p.fu.lex_mid_cnt[qi];
+    ovf = p.fu.lex_ovf[qi];
+    ovf_end = p.fu.q_indptr[qi + 1];
+#pragma unroll
+    for (int i = 0; i < kLexRegTerms; ++i) {
+      const int4 e = i < nreg ? p.fu.lex_terms[qi * kLexRegTerms + i] : make_int4(0, 0, 0, -1);
+      base[i] = cur[i] = e.x;
+      end[i] = e.y;
+      mul[i] = __int_as_float(e.z);
+      term[i] = e.w;
+    }
+#pragma unroll
+    for (int m = 0; m < kLexMidReg; ++m) {
+      const int2 e = m < nmid ? p.fu.lex_mid[qi * kLexMidReg + m] : make_int2(-1, 0);
+      mrow[m] = e.x;
+      mmul[m] = __int_as_float(e.y);
+    }
+    next_doc = -1;
+  }
+
+  // Places every tail cursor on the term's first posting with chunk >= d
+  // (interleaved binary searches: one load per term and step in flight).
+  __device__ __forceinline__ void seek(const int2* post, int64_t d) {
+    int lo[kLexRegTerms], hi[kLexRegTerms];
+#pragma unroll
+    for (int i = 0; i < kLexRegTerms; ++i) {
+      lo[i] = i < nreg ? base[i] : 0;
+      hi[i] = i < nreg ? end[i] : 0;
+    }
+    bool more = true;
+    while (more) {
+      int x[kLexRegTerms];
+#pragma unroll
+      for (int i = 0; i < kLexRegTerms; ++i)
+        x[i] = lo[i] < hi[i] ? __ldg(&post[(lo[i] + hi[i]) >> 1].x) : 0;
+      more = false;
+#pragma unroll
+      for (int i = 0; i < kLexRegTerms; ++i) {
+        if (lo[i] < hi[i]) {
+          const int mid = (lo[i] + hi[i]) >> 1;
+          if (x[i] < d) lo[i] = mid + 1; else hi[i] = mid;
+          more |= lo[i] < hi[i];
+        }
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < kLexRegTerms; ++i) cur[i] = lo[i];
+  }
+
+  // Copies the chunk's mid-row weights and the tail terms' next postings
+  // (chunks id0 .. id0 + 31) into the landing zone and waits for them.
+  __device__ __forceinline__ void fetch(const TcParams& p, int64_t id0, unsigned char* land) {
+    float* lm = reinterpret_cast<float*>(land);
+    int2* lt = reinterpret_cast<int2*>(land + kLexMidReg * 128);
+#pragma unroll
+    for (int m = 0; m < kLexMidReg; ++m) {
+      if (m < nmid) {
+        const float* src = p.fu.mid_w + static_cast<int64_t>(mrow[m]) * p.fu.mid_ld + id0;
+#pragma unroll
+        for (int g = 0; g < 8; ++g) cp_async16(lm + m * 32 + 4 * g, src + 4 * g);
+      }
+    }
+    const int2* post = p.fu.lex_post;
+#pragma unroll
+    for (int i = 0; i < kLexRegTerms; ++i) {
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        if (i < nreg && cur[i] + u < end[i]) cp_async8(lt + 2 * i + u, post + cur[i] + u);
+        else lt[2 * i + u] = make_int2(0x7FFFFFFF, 0);
+      }
+    }
+    cp_async_commit_wait_all();
+  }
+
+  // The chunk's mid-row part of element i (landing zone filled by fetch).
+  __device__ __forceinline__ float4 mid4(const unsigned char* land, int g) const {
+    const float* lm = reinterpret_cast<const float*>(land);
+    float4 r = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int m = 0; m < kLexMidReg; ++m) {
+      if (m < nmid) {
+        const float4 x = *reinterpret_cast<const float4*>(lm + m * 32 + 4 * g);
+        r.x = fmaf(mmul[m], x.x, r.x);
+        r.y = fmaf(mmul[m], x.y, r.y);
+        r.z = fmaf(mmul[m], x.z, r.z);
+        r.w = fmaf(mmul[m], x.w, r.w);
+      }
+    }
+    return r;
+  }
+
+  // Adds the chunk's tail-term (and long-query) BM25 into the thread's
+  // staging row (float4 groups XOR-swizzled by swz), which holds zeros on
+  // entry, and advances the tail cursors past the chunk.
+  __device__ __forceinline__ void tail(const TcParams& p, int64_t id0, const unsigned char* land,
+                                       float* srow, int swz) {
+    const int2* post = p.fu.lex_post;
+    const int2* lt = reinterpret_cast<const int2*>(land + kLexMidReg * 128);
+    const int64_t lim = id0 + 32;
+    auto add = [&](int2 e, float m) {
+      const int i = static_cast<int>(e.x - id0);
+      srow[((((i & 31) >> 2) ^ swz) << 2) | (i & 3)] += m * __int_as_float(e.y);
+    };
+#pragma unroll
+    for (int i = 0; i < kLexRegTerms; ++i) {
+      const int2 e0 = lt[2 * i], e1 = lt[2 * i + 1];
+      if (e0.x < lim) {
+        add(e0, mul[i]);
+        int c = cur[i] + 1;
+        if (e1.x < lim) {
+          add(e1, mul[i]);
+          ++c;
+          while (c < end[i]) {
+            const int2 e = __ldg(post + c);
+            if (e.x >= lim) break;
+            add(e, mul[i]);
+            ++c;
+          }
+        }
+        cur[i] = c;
+      }
+    }
+    // Further terms of a long query (each occurrence once): mid rows read
+    // directly, tail terms by a binary search per chunk.
+    for (int j = ovf; j < ovf_end; ++j) {
+      const int32_t tm = p.fu.q_terms[j];
+      if (tm < 0 || tm >= p.fu.vocab) continue;
+      const int cls = p.fu.lex_class[tm];
+      if (cls >= 0) continue;
+      if (cls <= -2) {
+        bool listed = false;
+#pragma unroll
+        for (int m = 0; m < kLexMidReg; ++m) listed |= m < nmid && mrow[m] == -2 - cls;
+        if (listed) continue;
+        const float* row = p.fu.mid_w + static_cast<int64_t>(-2 - cls) * p.fu.mid_ld + id0;
+        for (int i = 0; i < 32; ++i) srow[(((i >> 2) ^ swz) << 2) | (i & 3)] += __ldg(row + i);
+        continue;
+      }
+      bool listed = false;
+#pragma unroll
+      for (int i = 0; i < kLexRegTerms; ++i) listed |= term[i] == tm;
+      if (listed) continue;
+      int lo = static_cast<int>(p.fu.post_ptr[tm]);
+      const int stop = static_cast<int>(p.fu.post_ptr[tm + 1]);
+      int hi = stop;
+      while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (__ldg(&post[mid].x) < id0) lo = mid + 1; else hi = mid;
+      }
+      for (; lo < stop; ++lo) {
+        const int2 e = __ldg(post + lo);
+        if (e.x >= lim) break;
+        add(e, 1.f);
+      }
+    }
+  }
+};
+
 // ----------------------------------------------------------------- kernel
 
 // kPair: the grid is made of clusters of two CTAs that share every unit: a
@@ -623,18 +837,36 @@ struct EpiList<K, true> {
 // Epilogue set s filters query tile 2J + s, so one unit's epilogue overlaps
 // the next unit's copies and MMAs.  Per unit the CTA reads the corpus tile
 // once for 256 queries.
-template <int BN, int K, bool kHybrid, bool kPair = false, bool kDual = false>
-__global__ void __launch_bounds__(threads_for(K), 1)
+//
+// kLex: the lexical part of the hybrid search (Sec. 4.4 fusion).
+// kLexNone: dense scores.  kLexBlock: the epilogue reads BM25(q, d) from the
+// q x ld block that the BM25 pass materialised.  kLexGather (single CTAs,
+// BN = 128, one epilogue set): the gathered hybrid
+// search.  After the unit's score K blocks the producer loads one more stage,
+// the query tile's head-term counts (map_qb) and the corpus tile's split
+// head-term weights (map_eb), and the MMA issuer accumulates their product
+// into a second accumulator (the head terms' BM25, columns 2 BN + acc BN);
+// the epilogue adds the other terms from the postings (LexCursor) and fuses.
+constexpr int kLexNone = 0, kLexBlock = 1, kLexGather = 2;
+
+template <int BN, int K, int kLex, bool kPair = false, bool kDual = false>
+__global__ void __launch_bounds__(threads_for(K, kLex == kLexGather), 1)
 tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_e,
-                 const TcParams p) {
+                 const __grid_constant__ CUtensorMap map_qb,
+                 const __grid_constant__ CUtensorMap map_eb, const TcParams p) {
   static_assert(!(kPair && kDual), "pair and dual modes are exclusive");
   static_assert(!kDual || epi_sets(K) == 2, "dual mode needs one epilogue set per query tile");
   static_assert(!kDual || BN == 128, "dual mode double-buffers four accumulators of 128 columns");
-  constexpr int S = stages_for<BN, kPair, kDual>();
+  constexpr bool kHybrid = kLex == kLexGather;   // the gathered form
+  static_assert(!kHybrid || (!kPair && !kDual && BN == 128),
+                "the gathered hybrid search runs single CTAs on 128-row tiles");
+  constexpr int S = stages_for<BN, kPair, kDual, kHybrid>();
   constexpr uint32_t kAStage = a_stage_bytes<kDual>();
   constexpr uint32_t kBStageBytes = b_stage_bytes<BN, kPair>();
-  constexpr uint32_t kTmemCols = (kDual ? 4 : 2) * BN;
-  constexpr int kEpiSets = epi_sets(K);
+  constexpr uint32_t kTmemCols = (kDual ? 4 : 2) * BN * (kHybrid ? 2 : 1);
+  constexpr int kEpiSets = epi_sets(K, kHybrid);
+  // Stages per unit: the score K blocks, plus the head-term block (hybrid).
+  const int unit_kb = p.kblocks + (kHybrid ? 1 : 0);
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   if (threadIdx.x == 0) note_phase(p, kPhEntry);
   unsigned char* base = reinterpret_cast<unsigned char*>(
@@ -642,7 +874,9 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
   unsigned char* sA = base;
   unsigned char* sB = sA + S * kAStage;
   float* stage_rows = reinterpret_cast<float*>(sB + S * kBStageBytes);   // epilogue staging
-  uint64_t* full = reinterpret_cast<uint64_t*>(stage_rows + kEpiSets * 128 * 32);
+  // hybrid: each epilogue thread's landing zone of the lexical copies
+  unsigned char* lex_land = reinterpret_cast<unsigned char*>(stage_rows + kEpiSets * 128 * 32);
+  uint64_t* full = reinterpret_cast<uint64_t*>(lex_land + lex_land_bytes(kHybrid));
   uint64_t* empty = full + S;
   uint64_t* tfull = empty + S;
   uint64_t* tempty = tfull + 4;
@@ -681,6 +915,10 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     fence_mbar_init();
     prefetch_map(&map_q);
     prefetch_map(&map_e);
+    if constexpr (kHybrid) {
+      prefetch_map(&map_qb);
+      prefetch_map(&map_eb);
+    }
   }
   // The peer's copies and arrivals target the leader's barriers: both CTAs'
   // barriers are initialised before either CTA issues anything.
@@ -691,6 +929,11 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       const uint32_t bar = cluster_addr(&full[s], 0);                  // the leader's full[s]
       tma_load_2d_pair(sA + s * kAStage, &map_q, bar, kb * kBlockK, a_row(J));
       tma_load_2d_pair(sB + s * kBStageBytes, &map_e, bar, kb * kBlockK, b_row(t));
+    } else if (kHybrid && kb == p.kblocks) {
+      // the head-term stage: counts x split weights (one 64-element K block)
+      mbar_arrive_expect_tx(&full[s], stage_tx);
+      tma_load_2d(sA + s * kAStage, &map_qb, &full[s], 0, a_row(J));
+      tma_load_2d(sB + s * kBStageBytes, &map_eb, &full[s], 0, b_row(t));
     } else {
       mbar_arrive_expect_tx(&full[s], stage_tx);
       tma_load_2d(sA + s * kAStage, &map_q, &full[s], kb * kBlockK, a_row(J));
@@ -706,7 +949,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     UnitSeq us;
     us.start(p, cta, C);
     for (; us.valid() && pre_issued < S; us.next()) {
-      for (int kb = 0; kb < p.kblocks && pre_issued < S; ++kb, ++pre_issued)
+      for (int kb = 0; kb < unit_kb && pre_issued < S; ++kb, ++pre_issued)
         load_stage(pre_issued, kb, us.j(), us.t());
       if (pre_issued >= S) break;
     }
@@ -736,7 +979,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       for (us.start(p, cta, C); ok && us.valid(); us.next()) {
         const int j = us.j();
         const int t = us.t();
-        for (int kb = 0; kb < p.kblocks; ++kb) {
+        for (int kb = 0; kb < unit_kb; ++kb) {
           if (skip > 0) {
             --skip;
             issued |= 1u << s;
@@ -806,7 +1049,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         if (!mbar_wait<kPair>(&tempty[acc], acc_ph ^ 1u, abort_flag, p.dev_err, p.wait_limit)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
-        for (int kb = 0; kb < p.kblocks; ++kb) {
+        for (int kb = 0; kb < unit_kb; ++kb) {
           if (!mbar_wait(&full[s], ph, abort_flag, p.dev_err, p.wait_limit)) { ok = false; break; }
           tc_fence_after();
           if (p.phases != nullptr) {
@@ -816,7 +1059,14 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
           }
           const uint64_t a = sw128_desc(smem_addr(sA + s * kAStage));
           const uint64_t b = sw128_desc(smem_addr(sB + s * kBStageBytes));
-          if constexpr (kPair) {
+          if (kHybrid && kb == p.kblocks) {
+            // head-term BM25 of the unit into the second accumulator
+            const uint32_t d_lex = tmem_base + static_cast<uint32_t>((2 + acc) * BN);
+#pragma unroll
+            for (int kk = 0; kk < kBlockK / kUmmaK; ++kk)
+              mma_bf16(d_lex, a + 2 * kk, b + 2 * kk, idesc, kk != 0 ? 1u : 0u);
+            mma_commit(&empty[s]);
+          } else if constexpr (kPair) {
 #pragma unroll
             for (int kk = 0; kk < kBlockK / kUmmaK; ++kk)
               mma_bf16_pair(d_tmem, a + 2 * kk, b + 2 * kk, idesc, (kb | kk) != 0 ? 1u : 0u);
@@ -867,6 +1117,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     EpiList<K> list;
     list.set_k(p.k);
     list.clear();
+    LexCursor lex;             // hybrid: the query's postings cursors
 
     // This CTA owns the list slots (J, cta - first_cta(J)); empty them first.
     for (int J = 0; J < p.qt; ++J) {
@@ -900,8 +1151,17 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         cur_valid = valid && owns(J);
         if (cur_valid) list.load(p, cur_sr); else list.clear();
         if constexpr (K > 32) list.set_query(p, static_cast<int64_t>(j) * kBlockM + row, cur_valid);
+        if constexpr (kHybrid) {
+          if (cur_valid) lex.set_query(p, static_cast<int64_t>(j) * kBlockM + row);
+        }
       }
       const bool act = cur_valid;
+      if constexpr (kHybrid) {
+        // Place the postings cursors at this unit's first chunk (while its
+        // MMAs run) unless they continue from the previous unit.
+        if (act && lex.next_doc != t * BN) lex.seek(p.fu.lex_post, t * BN);
+        lex.next_doc = (t + 1) * BN;
+      }
       // Shared bound of this query's k-th best score, read while the MMAs run.
       float gfl = -INFINITY;
       if constexpr (K <= 32) {
@@ -919,10 +1179,10 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       if (warp_live) {
         float inv_max = 0.f;
         const float* brow = nullptr;
-        if (kHybrid && act) {
+        if (kLex != kLexNone && act) {
           const float m = p.fu.bm25_max[j * kBlockM + row];
           inv_max = m > 0.f ? 1.f / m : 0.f;
-          brow = p.fu.bm25 + static_cast<int64_t>(j * kBlockM + row) * p.fu.ld;
+          if (kLex == kLexBlock) brow = p.fu.bm25 + static_cast<int64_t>(j * kBlockM + row) * p.fu.ld;
         }
         const uint32_t taddr = tmem_base + (static_cast<uint32_t>(eg * 32) << 16) +
                                static_cast<uint32_t>(acc * BN);
@@ -930,27 +1190,62 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         // that the 32 lanes' 16-byte stores spread over all banks.
         float* srow = stage_rows + ((warp - 2) * 32 + lane) * 32;
         const int swz = lane & 7;
+        unsigned char* land = lex_land + ((warp - 2) * 32 + lane) * kLexLandStride;
         // Scores of one chunk (corpus rows id0 .. id0 + 31), fused with the
-        // lexical part when hybrid, -inf past the end of the corpus.
+        // lexical part when hybrid, -inf past the end of the corpus.  Called
+        // by every lane of a live warp (the TMEM load is warp-collective).
         auto scores = [&](const uint32_t (&r)[32], int c, float (&v)[32]) {
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
           const int64_t id0 = t * BN + c * 32;
-          if (kHybrid && act) {
-            const float a = p.fu.alpha, b1 = 1.f - p.fu.alpha;
-            if (id0 + 32 <= p.n) {
+          if constexpr (kLex == kLexBlock) {
+            if (act) {
+              const float a = p.fu.alpha, b1 = 1.f - p.fu.alpha;
+              if (id0 + 32 <= p.n) {
 #pragma unroll
-              for (int i = 0; i < 32; i += 4) {
-                const float4 w = *reinterpret_cast<const float4*>(brow + id0 + i);
-                v[i] = fmaf(a, v[i], b1 * (w.x * inv_max));
-                v[i + 1] = fmaf(a, v[i + 1], b1 * (w.y * inv_max));
-                v[i + 2] = fmaf(a, v[i + 2], b1 * (w.z * inv_max));
-                v[i + 3] = fmaf(a, v[i + 3], b1 * (w.w * inv_max));
+                for (int i = 0; i < 32; i += 4) {
+                  const float4 w = *reinterpret_cast<const float4*>(brow + id0 + i);
+                  v[i] = fmaf(a, v[i], b1 * (w.x * inv_max));
+                  v[i + 1] = fmaf(a, v[i + 1], b1 * (w.y * inv_max));
+                  v[i + 2] = fmaf(a, v[i + 2], b1 * (w.z * inv_max));
+                  v[i + 3] = fmaf(a, v[i + 3], b1 * (w.w * inv_max));
+                }
+              } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i)
+                  if (id0 + i < p.n) v[i] = fmaf(a, v[i], b1 * (brow[id0 + i] * inv_max));
               }
-            } else {
+            }
+          }
+          if constexpr (kHybrid) {
+            // head terms from the second accumulator, the other terms from
+            // the postings (gathered into the staging row while the TMEM
+            // load is in flight), then the Sec. 4.4 weighted fusion
+            uint32_t rl[32];
+            tmem_ld32_async(taddr + 2 * BN + c * 32, rl);
+            if (act) {
+              lex.fetch(p, id0, land);
 #pragma unroll
-              for (int i = 0; i < 32; ++i)
-                if (id0 + i < p.n) v[i] = fmaf(a, v[i], b1 * (brow[id0 + i] * inv_max));
+              for (int g = 0; g < 8; ++g)
+                *reinterpret_cast<float4*>(srow + (g << 2)) = make_float4(0.f, 0.f, 0.f, 0.f);
+              lex.tail(p, id0, land, srow, swz);
+            }
+            tmem_wait_ld(rl);
+            if (act) {
+              const float a = p.fu.alpha, b1 = 1.f - p.fu.alpha;
+#pragma unroll
+              for (int g = 0; g < 8; ++g) {
+                const float4 x = *reinterpret_cast<const float4*>(srow + ((g ^ swz) << 2));
+                const float4 y = lex.mid4(land, g);
+                v[4 * g] = fmaf(
+                    a, v[4 * g], b1 * ((__uint_as_float(rl[4 * g]) + x.x + y.x) * inv_max));
+                v[4 * g + 1] = fmaf(
+                    a, v[4 * g + 1], b1 * ((__uint_as_float(rl[4 * g + 1]) + x.y + y.y) * inv_max));
+                v[4 * g + 2] = fmaf(
+                    a, v[4 * g + 2], b1 * ((__uint_as_float(rl[4 * g + 2]) + x.z + y.z) * inv_max));
+                v[4 * g + 3] = fmaf(
+                    a, v[4 * g + 3], b1 * ((__uint_as_float(rl[4 * g + 3]) + x.w + y.w) * inv_max));
+              }
             }
           }
           if (id0 + 32 > p.n) {
@@ -1001,7 +1296,9 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         static_assert(NC % 2 == 0, "chunks are processed in pairs");
         uint32_t ra[32], rb[32];
         float bound = -INFINITY;
-        if constexpr (K <= 32) {
+        // (Hybrid: no group bound for a fresh list, whose scores would need
+        // a second walk of the postings.)
+        if constexpr (K <= 32 && !kHybrid) {
           if (__any_sync(0xffffffffu, act && !list.full())) {
             // A list that is not full yet would take almost every score of
             // this unit as a candidate.  Cut the unit's columns into groups:
@@ -1123,14 +1420,20 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
 
 // ----------------------------------------------------------------- launch
 
+// Tensor maps of one launch: queries and corpus (score K blocks), and for the
+// gathered hybrid search the head-term counts and split weights (otherwise
+// copies of the first two, unused).
+struct TcMaps {
+  CUtensorMap q, e, qb, eb;
+};
+
 // Pair mode: clusters of two CTAs; `grid` counts CTAs (even).
-template <int BN, int K, bool H>
-cudaError_t launch_pair_variant(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
-                                int grid, cudaStream_t st) {
+template <int BN, int K, int L>
+cudaError_t launch_pair_variant(const TcMaps& m, const TcParams& prm, int grid, cudaStream_t st) {
   constexpr size_t smem = smem_for<BN, K, true>();
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(tc_search_kernel<BN, K, H, true>,
+    cudaError_t e = cudaFuncSetAttribute(tc_search_kernel<BN, K, L, true>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
@@ -1148,78 +1451,86 @@ cudaError_t launch_pair_variant(const CUtensorMap& mq, const CUtensorMap& me, co
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, tc_search_kernel<BN, K, H, true>, mq, me, prm);
+  return cudaLaunchKernelEx(&cfg, tc_search_kernel<BN, K, L, true>, m.q, m.e, m.qb, m.eb, prm);
 }
 
 // Clusters of two CTAs of a pair-mode search kernel that fit on the device at
 // once (the kernels' shared-memory use keeps one CTA per SM).
 int pair_capacity_query();
 
-template <int BN, int K, bool H>
-cudaError_t launch_variant(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
-                           int grid, cudaStream_t st) {
-  constexpr size_t smem = smem_for<BN, K>();
+template <int BN, int K, int L>
+cudaError_t launch_variant(const TcMaps& m, const TcParams& prm, int grid, cudaStream_t st) {
+  constexpr bool g = L == kLexGather;
+  constexpr size_t smem = smem_for<BN, K, false, false, g>();
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(tc_search_kernel<BN, K, H>,
+    cudaError_t e = cudaFuncSetAttribute(tc_search_kernel<BN, K, L>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  tc_search_kernel<BN, K, H><<<grid, threads_for(K), smem, st>>>(mq, me, prm);
+  tc_search_kernel<BN, K, L><<<grid, threads_for(K, g), smem, st>>>(m.q, m.e, m.qb, m.eb, prm);
   return cudaGetLastError();
 }
 
 // Dual mode (two query tiles per unit); 128-row corpus tiles, lists of 8 or 16.
-template <int K, bool H>
-cudaError_t launch_dual_variant(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
-                                int grid, cudaStream_t st) {
+template <int K, int L>
+cudaError_t launch_dual_variant(const TcMaps& m, const TcParams& prm, int grid, cudaStream_t st) {
   constexpr size_t smem = smem_for<128, K, false, true>();
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(tc_search_kernel<128, K, H, false, true>,
+    cudaError_t e = cudaFuncSetAttribute(tc_search_kernel<128, K, L, false, true>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  tc_search_kernel<128, K, H, false, true><<<grid, threads_for(K), smem, st>>>(mq, me, prm);
+  tc_search_kernel<128, K, L, false, true><<<grid, threads_for(K), smem, st>>>(m.q, m.e, m.qb,
+                                                                               m.eb, prm);
   return cudaGetLastError();
 }
 
-template <int BN, int K>
-cudaError_t launch_k(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm, int grid,
-                     bool hybrid, cudaStream_t st) {
-  return hybrid ? launch_variant<BN, K, true>(mq, me, prm, grid, st)
-                : launch_variant<BN, K, false>(mq, me, prm, grid, st);
+template <int BN, int L>
+cudaError_t launch_bn(const TcMaps& m, const TcParams& prm, int grid, cudaStream_t st) {
+  switch (list_len_for(prm.k)) {
+    case 8: return launch_variant<BN, 8, L>(m, prm, grid, st);
+    case 16: return launch_variant<BN, 16, L>(m, prm, grid, st);
+    case 32: return launch_variant<BN, 32, L>(m, prm, grid, st);
+    case 128: return launch_variant<BN, 128, L>(m, prm, grid, st);
+    default: return launch_variant<BN, 256, L>(m, prm, grid, st);
+  }
 }
 
-template <int BN>
-cudaError_t launch_bn(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm, int grid,
-                      bool hybrid, cudaStream_t st) {
+template <int L>
+cudaError_t launch_pair(const TcMaps& m, const TcParams& prm, int grid, cudaStream_t st) {
   switch (list_len_for(prm.k)) {
-    case 8: return launch_k<BN, 8>(mq, me, prm, grid, hybrid, st);
-    case 16: return launch_k<BN, 16>(mq, me, prm, grid, hybrid, st);
-    case 32: return launch_k<BN, 32>(mq, me, prm, grid, hybrid, st);
-    case 128: return launch_k<BN, 128>(mq, me, prm, grid, hybrid, st);
-    default: return launch_k<BN, 256>(mq, me, prm, grid, hybrid, st);
+    case 8: return launch_pair_variant<256, 8, L>(m, prm, grid, st);
+    case 16: return launch_pair_variant<256, 16, L>(m, prm, grid, st);
+    case 32: return launch_pair_variant<256, 32, L>(m, prm, grid, st);
+    case 128: return launch_pair_variant<256, 128, L>(m, prm, grid, st);
+    default: return launch_pair_variant<256, 256, L>(m, prm, grid, st);
+  }
+}
+
+template <int L>
+cudaError_t launch_dual(const TcMaps& m, const TcParams& prm, int grid, cudaStream_t st) {
+  switch (list_len_for(prm.k)) {
+    case 8: return launch_dual_variant<8, L>(m, prm, grid, st);
+    case 16: return launch_dual_variant<16, L>(m, prm, grid, st);
+    default: return cudaErrorInvalidValue;
   }
 }
 
 // Instantiations live in their own translation units (parallel builds).
-cudaError_t launch_bn128(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm, int grid,
-                        bool hybrid, cudaStream_t st);
-cudaError_t launch_bn256_dense(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
-                               int grid, cudaStream_t st);
-cudaError_t launch_bn256_fused(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
-                               int grid, cudaStream_t st);
-cudaError_t launch_pair256_dense(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
-                                 int grid, cudaStream_t st);
-cudaError_t launch_pair256_fused(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
-                                 int grid, cudaStream_t st);
-cudaError_t launch_dual128(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
-                           int grid, bool hybrid, cudaStream_t st);
+cudaError_t launch_bn128(const TcMaps& m, const TcParams& prm, int grid, int lex, cudaStream_t st);
+cudaError_t launch_bn128_gather(const TcMaps& m, const TcParams& prm, int grid, cudaStream_t st);
+cudaError_t launch_bn256_dense(const TcMaps& m, const TcParams& prm, int grid, cudaStream_t st);
+cudaError_t launch_bn256_block(const TcMaps& m, const TcParams& prm, int grid, cudaStream_t st);
+cudaError_t launch_pair256_dense(const TcMaps& m, const TcParams& prm, int grid, cudaStream_t st);
+cudaError_t launch_pair256_block(const TcMaps& m, const TcParams& prm, int grid, cudaStream_t st);
+cudaError_t launch_dual128(const TcMaps& m, const TcParams& prm, int grid, int lex,
+                           cudaStream_t st);
 
 }  // namespace tc
 }  // namespace oprag

@@ -4,15 +4,8 @@
 namespace oprag {
 namespace tc {
 
-cudaError_t launch_bn256_dense(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
-                               int grid, cudaStream_t st) {
-  switch (list_len_for(prm.k)) {
-    case 8: return launch_variant<256, 8, false>(mq, me, prm, grid, st);
-    case 16: return launch_variant<256, 16, false>(mq, me, prm, grid, st);
-    case 32: return launch_variant<256, 32, false>(mq, me, prm, grid, st);
-    case 128: return launch_variant<256, 128, false>(mq, me, prm, grid, st);
-    default: return launch_variant<256, 256, false>(mq, me, prm, grid, st);
-  }
+cudaError_t launch_bn256_dense(const TcMaps& m, const TcParams& prm, int grid, cudaStream_t st) {
+  return launch_bn<256, kLexNone>(m, prm, grid, st);
 }
 
 }  // namespace tc

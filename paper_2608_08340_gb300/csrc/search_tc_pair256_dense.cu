@@ -5,20 +5,13 @@
 namespace oprag {
 namespace tc {
 
-cudaError_t launch_pair256_dense(const CUtensorMap& mq, const CUtensorMap& me, const TcParams& prm,
-                                 int grid, cudaStream_t st) {
-  switch (list_len_for(prm.k)) {
-    case 8: return launch_pair_variant<256, 8, false>(mq, me, prm, grid, st);
-    case 16: return launch_pair_variant<256, 16, false>(mq, me, prm, grid, st);
-    case 32: return launch_pair_variant<256, 32, false>(mq, me, prm, grid, st);
-    case 128: return launch_pair_variant<256, 128, false>(mq, me, prm, grid, st);
-    default: return launch_pair_variant<256, 256, false>(mq, me, prm, grid, st);
-  }
+cudaError_t launch_pair256_dense(const TcMaps& m, const TcParams& prm, int grid, cudaStream_t st) {
+  return launch_pair<kLexNone>(m, prm, grid, st);
 }
 
 int pair_capacity_query() {
   constexpr size_t smem = smem_for<256, 16, true>();
-  if (cudaFuncSetAttribute(tc_search_kernel<256, 16, false, true>,
+  if (cudaFuncSetAttribute(tc_search_kernel<256, 16, kLexNone, true>,
                            cudaFuncAttributeMaxDynamicSharedMemorySize,
                            static_cast<int>(smem)) != cudaSuccess)
     return 0;
@@ -34,7 +27,7 @@ int pair_capacity_query() {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, tc_search_kernel<256, 16, false, true>, &cfg) !=
+  if (cudaOccupancyMaxActiveClusters(&n, tc_search_kernel<256, 16, kLexNone, true>, &cfg) !=
       cudaSuccess)
     return 0;
   return n;

@@ -235,6 +235,11 @@ class Index:
                                                  ctypes.byref(c)))
         return {"scratch": a.value, "bounds": b.value, "lexical": c.value}
 
+    def gather_lexical(self, on: bool = True) -> None:
+        """Hybrid search: gather BM25 in the search epilogue (True) instead of
+        reading a materialised q x n BM25 block (False, the default)."""
+        self.set_option(_lib.OPRAG_OPT_LEX_GATHER, int(on))
+
     PHASES = ("entry", "setup", "first_stage", "last_stage", "last_commit", "epi0_done",
               "epi1_done", "exit")
 

@@ -3,8 +3,10 @@ the exact dense top-N, then the fused rerank of only those candidates with
 the BM25 maximum taken over the candidates.  The rerank is checked against the
 oracle's rerank of the same candidates (the dense top-N itself is checked by
 the dense parity tests; near-ties at rank N could otherwise change the set),
-and with every chunk a candidate it must equal the full hybrid search bit for
-bit."""
+and with every chunk a candidate it must equal the full hybrid search: bit
+for bit with the materialised BM25 block (the same fp32 sums in query-term
+order), and up to the fp32 rounding of the sums with the gathered form (the
+head terms' part then comes from tensor-core MMAs)."""
 import numpy as np
 import pytest
 import torch
@@ -48,15 +50,23 @@ def test_dense_first_matches_oracle_rerank(n, q, n_cand, k):
     idx.check()
 
 
-def test_dense_first_over_every_chunk_equals_full_hybrid():
+@pytest.mark.parametrize("gather", [False, True])
+def test_dense_first_over_every_chunk_equals_full_hybrid(gather):
     w, idx = _setup(200, 50)
+    idx.gather_lexical(gather)
     qip, qt = _terms(w)
     Q = dev_tensor(w.Q_data)
-    d_ids, d_sc = idx.hybrid_search_dense_first(Q, qip, qt, w.alpha, 256, 10)
+    d_ids, d_sc = idx.hybrid_search_dense_first(Q, qip, qt, w.alpha, 256, 40)
     h_ids, h_sc = idx.hybrid_search(Q, qip, qt, w.alpha, 10)
     torch.cuda.synchronize()
-    assert torch.equal(d_ids, h_ids)
-    assert torch.equal(d_sc, h_sc)
+    if not gather:
+        assert torch.equal(d_ids[:, :10], h_ids)
+        assert torch.equal(d_sc[:, :10], h_sc)
+        return
+    # same ranking up to swaps of scores within 1e-5 (different fp32 sum orders)
+    check.check_topk(h_ids.cpu().numpy(), h_sc.cpu().numpy(), d_ids.cpu().numpy(),
+                     d_sc.cpu().numpy().astype(np.float64), 10, 1e-5, n=200,
+                     label="dense-first over every chunk vs gathered hybrid")
 
 
 def test_dense_first_alpha_one_is_the_dense_search():

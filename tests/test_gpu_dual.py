@@ -90,3 +90,25 @@ def test_dual_hybrid_matches_single():
     assert (res["dual"][1] - res["single"][1]).abs().max().item() <= TOL
     idx.check()
     idx.close()
+
+
+def test_gathered_hybrid_runs_single_ctas_whatever_the_pair_option():
+    """The gathered hybrid search (OPRAG_OPT_LEX_GATHER) takes every TMEM
+    column for two score and two BM25 accumulators, so it always runs single
+    CTAs on 128-row tiles; forcing dual mode changes nothing."""
+    w = workloads.config(3, n=6000, batch=300)
+    idx = Index(dev_tensor(w.E_data))
+    idx.set_sparse(w.doc_indptr, w.doc_terms, w.vocab, w.k1, w.b)
+    idx.force_path("tc")
+    idx.gather_lexical(True)
+    res = {}
+    for mode in ("dual", None):
+        idx.force_pair(mode)
+        res[mode] = idx.hybrid_search(dev_tensor(w.Q_data), torch.from_numpy(w.q_indptr),
+                                      torch.from_numpy(w.q_terms), w.alpha, w.k)
+        torch.cuda.synchronize()
+        assert idx.last_launch["tiles"] == 1 and idx.last_launch["block_n"] == 128
+    assert torch.equal(res["dual"][0], res[None][0])
+    assert torch.equal(res["dual"][1], res[None][1])
+    idx.check()
+    idx.close()

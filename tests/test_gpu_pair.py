@@ -83,3 +83,26 @@ def test_pair_hybrid_matches_single():
     assert (res["pair"][1] - res["single"][1]).abs().max().item() <= TOL
     idx.check()
     idx.close()
+
+
+def test_gathered_hybrid_ignores_pair_and_tile_options():
+    """The gathered hybrid search (OPRAG_OPT_LEX_GATHER) always runs single
+    CTAs on 128-row tiles
+    (its two score and two BM25 accumulators fill the TMEM); forcing CTA
+    pairs or 256-row tiles changes nothing."""
+    w = workloads.config(3, n=6000, batch=300)
+    idx = Index(dev_tensor(w.E_data))
+    idx.set_sparse(w.doc_indptr, w.doc_terms, w.vocab, w.k1, w.b)
+    idx.force_path("tc")
+    idx.gather_lexical(True)
+    res = {}
+    for mode, bn in (("pair", 256), (None, None)):
+        idx.force_block_n(bn)
+        idx.force_pair(mode)
+        res[mode] = idx.hybrid_search(dev_tensor(w.Q_data), torch.from_numpy(w.q_indptr),
+                                      torch.from_numpy(w.q_terms), w.alpha, w.k)
+        assert idx.last_launch["cluster"] == 1 and idx.last_launch["block_n"] == 128
+    assert torch.equal(res["pair"][0], res[None][0])
+    assert torch.equal(res["pair"][1], res[None][1])
+    idx.check()
+    idx.close()

@@ -94,8 +94,8 @@ def _csr(lists):
     return indptr, np.array([t for x in lists for t in x], np.int32)
 
 
-@pytest.mark.parametrize("path", ["simt", "tc"])
-def test_hybrid_golden_hand_worked(path):
+@pytest.mark.parametrize("path,gather", [("simt", False), ("tc", False), ("tc", True)])
+def test_hybrid_golden_hand_worked(path, gather):
     g = load("hybrid_4doc.json")
     bm = load("bm25_4doc.json")
     E = np.zeros((4, 8), np.float32)
@@ -106,19 +106,25 @@ def test_hybrid_golden_hand_worked(path):
     idx.force_path(path)
     dip, dt = _csr(bm["docs"])
     idx.set_sparse(dip, dt, bm["vocab"], bm["k1"], bm["b"])
+    idx.gather_lexical(gather)
     qip, qt = _csr(g["query_terms"])
     ids, sc = idx.hybrid_search(dev_tensor(oracle.round_bf16(Q)), torch.from_numpy(qip),
                                 torch.from_numpy(qt), g["alpha"], g["k"])
     want = np.array([[value(x) for x in r] for r in g["scores"]])
-    np.testing.assert_allclose(sc.cpu().numpy(), want, atol=1e-6)
+    # Materialised block: fp32 sums of the exact fp32 weights.  Gathered: a
+    # head term's weight enters the tensor cores as a high + low bf16 pair,
+    # within 2^-18 of it relatively, so the lexical half (1 - alpha) BM25 / max
+    # is within about 2e-6.
+    np.testing.assert_allclose(sc.cpu().numpy(), want, atol=1e-5 if gather else 1e-6)
     got = ids.cpu().tolist()
     assert got[0][0] == 0 and sorted(got[0][1:3]) == [1, 2] and got[0][3] == 3
     assert sorted(got[1][:2]) == [1, 2] and sorted(got[1][2:]) == [0, 3]
 
 
-def _hybrid_check(idx, w, rows, alpha, label):
+def _hybrid_check(idx, w, rows, alpha, label, k=None):
+    k = k or w.k
     ids, sc = idx.hybrid_search(dev_tensor(w.Q_data), torch.from_numpy(w.q_indptr),
-                                torch.from_numpy(w.q_terms), alpha, w.k)
+                                torch.from_numpy(w.q_terms), alpha, k)
     ids = ids.cpu().numpy()[rows]
     sc = sc.cpu().numpy()[rows]
     qip = np.zeros(len(rows) + 1, np.int32)
@@ -128,8 +134,8 @@ def _hybrid_check(idx, w, rows, alpha, label):
     o_ids, o_sc = oracle_topk(
         lambda kout: oracle.hybrid_search(w.E_data, w.Q_data[rows], w.doc_indptr, w.doc_terms,
                                           w.vocab, qip, qt, alpha, kout, w.k1, w.b),
-        w.k, w.n)
-    return check.check_topk(ids, sc, o_ids, o_sc, w.k, TOL, n=w.n, label=label,
+        k, w.n)
+    return check.check_topk(ids, sc, o_ids, o_sc, k, TOL, n=w.n, label=label,
                             query_index=rows)
 
 
@@ -141,10 +147,16 @@ def cfg3():
     return w, idx
 
 
-def test_config3_hybrid_every_query(cfg3):
-    """All 1024 queries of the hybrid workload against the oracle."""
+@pytest.mark.parametrize("gather", [False, True])
+def test_config3_hybrid_every_query(cfg3, gather):
+    """All 1024 queries of the hybrid workload against the oracle, with the
+    BM25 block and with the BM25 gathered in the search epilogue."""
     w, idx = cfg3
-    _hybrid_check(idx, w, np.arange(w.q), w.alpha, "cfg3")
+    idx.gather_lexical(gather)
+    try:
+        _hybrid_check(idx, w, np.arange(w.q), w.alpha, f"cfg3 gather={gather}")
+    finally:
+        idx.gather_lexical(False)
     assert idx.last_path == "tc"
     idx.check()
 
@@ -178,3 +190,86 @@ def test_hybrid_without_sparse_side_is_not_ready():
         idx.hybrid_search(dev_tensor(w.Q_data), torch.tensor([0, 1, 2]), torch.tensor([1, 2]),
                           0.5, 5)
     assert "NOT_READY" in str(e.value)
+
+
+# ---------------------------------------------------------------- both forms
+# With OPRAG_OPT_LEX_GATHER the lexical part is gathered in the search
+# epilogue: the 32 commonest terms through tensor-core MMAs of counts x split
+# weights, terms in at least 1/32 of the chunks as fp32 rows (2 per query in
+# the landing zone, further ones read directly), the others from their
+# postings with per-thread cursors (up to 8 distinct terms), any further
+# terms of a long query by a per-chunk search.  Each case runs both forms.
+
+
+@pytest.mark.parametrize("gather", [False, True])
+def test_hybrid_long_queries_with_repeats_and_many_terms(gather):
+    """12-40 terms per query: more than 8 distinct postings terms (the
+    overflow scan), repeated terms and head terms mixed in."""
+    w = workloads.config(3, n=6000, batch=40)
+    rng = np.random.default_rng(11)
+    lists = []
+    for i in range(w.q):
+        tail = rng.integers(30, 3000, size=int(rng.integers(12, 41))).tolist()
+        head = rng.integers(0, 12, size=3).tolist()
+        t = tail + head + tail[:4]                  # the first four tail terms twice
+        rng.shuffle(t)
+        lists.append(t)
+    w.q_indptr, w.q_terms = _csr(lists)
+    idx = Index(dev_tensor(w.E_data))
+    idx.set_sparse(w.doc_indptr, w.doc_terms, w.vocab, w.k1, w.b)
+    idx.gather_lexical(gather)
+    _hybrid_check(idx, w, np.arange(w.q), w.alpha, f"long queries gather={gather}")
+    assert idx.last_path == "tc"
+    idx.check()
+
+
+@pytest.mark.parametrize("gather", [False, True])
+def test_hybrid_more_head_terms_than_tensor_core_slots(gather):
+    """60 terms occur in most chunks: the 32 commonest are scored on tensor
+    cores, the other 28 through their postings."""
+    rng = np.random.default_rng(12)
+    n, vocab = 3000, 500
+    bags = []
+    for _ in range(n):
+        common = [t for t in range(60) if rng.random() < 0.85] * int(rng.integers(1, 3))
+        bags.append(common + rng.integers(60, vocab, size=int(rng.integers(20, 60))).tolist())
+    w = workloads.config(3, n=n, batch=70)
+    w.doc_indptr, w.doc_terms = _csr(bags)
+    w.vocab = vocab
+    lists = [rng.integers(0, 60, size=5).tolist() + rng.integers(60, vocab, size=4).tolist()
+             for _ in range(w.q)]
+    w.q_indptr, w.q_terms = _csr(lists)
+    idx = Index(dev_tensor(w.E_data))
+    idx.set_sparse(w.doc_indptr, w.doc_terms, w.vocab, w.k1, w.b)
+    idx.gather_lexical(gather)
+    for alpha in (w.alpha, 0.0):
+        _hybrid_check(idx, w, np.arange(w.q), alpha, f"60 head terms alpha={alpha}")
+
+
+@pytest.mark.parametrize("gather", [False, True])
+@pytest.mark.parametrize("k", [33, 100])
+def test_hybrid_large_k_with_sampled_floor(k, gather):
+    """k > 32 over 313 corpus tiles: the sampled first pass (every 32nd tile,
+    so the postings cursors are placed again at every unit) runs the fused
+    epilogue too."""
+    w = workloads.config(3, n=40000, batch=130)
+    idx = Index(dev_tensor(w.E_data))
+    idx.set_sparse(w.doc_indptr, w.doc_terms, w.vocab, w.k1, w.b)
+    idx.gather_lexical(gather)
+    idx.enable_timing(True)
+    rows = np.sort(np.random.default_rng(k).choice(w.q, 24, replace=False))
+    _hybrid_check(idx, w, rows, w.alpha, f"hybrid k={k}", k=k)
+    assert idx.last_timing()["sample_ms"] > 0.0
+    idx.check()
+
+
+@pytest.mark.parametrize("gather", [False, True])
+@pytest.mark.parametrize("n,q,k", [(9000, 300, 16), (129, 5, 7), (4500, 257, 1)])
+def test_hybrid_ragged_tiles(n, q, k, gather):
+    """Ragged corpus and query tiles, several query tiles per CTA."""
+    w = workloads.config(3, n=n, batch=q)
+    idx = Index(dev_tensor(w.E_data))
+    idx.set_sparse(w.doc_indptr, w.doc_terms, w.vocab, w.k1, w.b)
+    idx.gather_lexical(gather)
+    _hybrid_check(idx, w, np.arange(w.q), w.alpha, f"ragged n={n} q={q} k={k} gather={gather}", k=k)
+    idx.check()
