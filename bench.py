@@ -911,10 +911,13 @@ def run_index_ops(args):
     idx.close()
     # knowledge (32768) + memory (8192) search of 256 queries against knowledge alone
     kn = Index(to_dev(w.E_data))
-    mem = Index(to_dev(workloads.config(1, n=8192, batch=1).E_data))
+    mem_rows = workloads.config(1, n=8192, batch=1).E_data
+    mem = Index(to_dev(mem_rows))
+    stacked = Index(to_dev(np.concatenate([w.E_data, mem_rows])))
     Q = to_dev(workloads.config(1, batch=256).Q_data)
     for label, fn in (("search_knowledge_ms", lambda: kn.search(Q, w.k)),
-                      ("search_two_ms", lambda: search_two(kn, mem, Q, w.k))):
+                      ("search_two_ms", lambda: search_two(kn, mem, Q, w.k)),
+                      ("search_stacked_40960_ms", lambda: stacked.search(Q, w.k))):
         for _ in range(args.warmup):
             fn()
         marks = []

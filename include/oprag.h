@@ -227,12 +227,16 @@ OPRAG_API int oprag_index_update_sparse(oprag_index *idx, const int64_t *ids, in
                                         const int32_t *bag_indptr, const int32_t *bag_terms);
 
 /*
- * Dense top-k over a knowledge index and a memory index together (Sec. 4.4:
- * both indices are searched the same way; one ranked result).  Same dim and
- * dtype on the same device.  out_ids: chunk id within its index; out_src: 0 =
- * knowledge, 1 = memory (device, q x k each, out_scores as oprag_search).
- * Order: score descending, then knowledge before memory, then chunk id.
- * k <= n_knowledge + n_memory.  Asynchronous on `stream`.
+ * Dense top-k over a knowledge index and a memory index together (Sec. 3.6,
+ * Sec. 4.4: both indices are searched the same way; one ranked result).  Same
+ * dim and dtype on the same device.  out_ids: chunk id within its index;
+ * out_src: 0 = knowledge, 1 = memory (device, q x k each, out_scores as
+ * oprag_search).  Order: score descending, then knowledge before memory, then
+ * chunk id.  k <= n_knowledge + n_memory.  Asynchronous on `stream`.
+ * bf16 indices: one launch of the search kernel scans the knowledge rows
+ * followed by the memory rows (plus its sampled first pass when k > 32 over
+ * many tiles) and one merge writes the result, using the knowledge index's
+ * scratch; fp32 indices: a search per index and a merge of the two lists.
  */
 OPRAG_API int oprag_search_two(oprag_index *knowledge, oprag_index *memory, const void *queries,
                                int32_t q, int32_t k, int64_t *out_ids, int32_t *out_src,

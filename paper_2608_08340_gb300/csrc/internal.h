@@ -33,6 +33,11 @@ struct ListSet {
   int sets = 1;
   int pair = 1;
   int klen = 1 << 30;   // sorted keys held per list (the merge reads min(k, klen))
+  // Search over two stacked corpora (oprag_search_two): ids >= split belong
+  // to the second; the merge then writes id - split and out_src = 1 (else
+  // the id and 0; -1 for an empty result).  out_src == nullptr: ids as kept.
+  int64_t split = 0;
+  int32_t* out_src = nullptr;
 };
 
 // Optional lexical part of the fused score (Sec. 4.4 weighted fusion):
@@ -87,6 +92,9 @@ struct SearchShape {
   int d;
   int q;
   int k;
+  // Rows of a second corpus searched after the first in the same launch
+  // (its chunks get ids n + row); 0 for one corpus.
+  int64_t n_second = 0;
   // The lexical part is gathered in the tensor-core epilogue: the plan uses
   // single CTAs with 128-row corpus tiles and one epilogue set.
   bool fused_lex = false;
@@ -102,6 +110,7 @@ cudaError_t launch_simt_search(int dtype, const void* E, const void* Q, const Se
 // --- tcgen05 tensor-core search (bf16).
 struct TcPlan {
   int block_n;     // corpus rows per tile: 128 or 256
+  int nt_first;    // corpus tiles of the first corpus (nt_first == tiles of all when one)
   int grid;        // CTAs (persistent)
   int pair;        // 2: clusters of two CTAs issue M = 256 MMAs together; 1: single CTAs
   bool dual;       // single CTAs that take two query tiles per unit (see search_tc.cuh)
@@ -136,12 +145,14 @@ size_t tc_scratch_bytes(const SearchShape& s, const TcPlan& p);
 // phases (optional, grid x kTcPhases zeroed words): global-timer stamps of
 // each CTA's run (entry, setup done, first and last stage landed, last MMA
 // commit, epilogue sets done, exit), for measurement.
+// E2 (s.n_second > 0): the second corpus, same d and dtype.
 cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s, const Fusion& fu,
                              const TcPlan& plan, void* scratch, int* dev_err, ListSet* lists,
                              cudaStream_t st, const float* init_floor = nullptr,
                              uint64_t* qfloor = nullptr, uint32_t gen = 0,
                              const float* levels = nullptr, int* level_cnt = nullptr,
-                             long long wait_limit = 0, unsigned long long* phases = nullptr);
+                             long long wait_limit = 0, unsigned long long* phases = nullptr,
+                             const void* E2 = nullptr);
 constexpr int kTcPhases = 8;
 
 // --- final merge of partial lists into the sorted top-k per query.

@@ -100,8 +100,7 @@ merge_kway_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
       const int i = (r & ~31) + lane;
       if (i <= r) {
         const int64_t o = static_cast<int64_t>(qi) * k + i;
-        out_ids[o] = mine == kEmptyKey ? -1 : static_cast<int64_t>(key_id(mine));
-        out_scores[o] = mine == kEmptyKey ? -INFINITY : key_score(mine);
+        store_result(ls, out_ids, out_scores, o, mine);
       }
     }
     if (r == k - 1 && kth_out != nullptr && lane == 0)
@@ -199,8 +198,7 @@ merge_small_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
       const int i = (r & ~31) + lane;
       if (i <= r) {
         const int64_t o = static_cast<int64_t>(qi) * k + i;
-        out_ids[o] = mine == kEmptyKey ? -1 : static_cast<int64_t>(key_id(mine));
-        out_scores[o] = mine == kEmptyKey ? -INFINITY : key_score(mine);
+        store_result(ls, out_ids, out_scores, o, mine);
       }
     }
     if (r == k - 1 && kth_out != nullptr && lane == 0)

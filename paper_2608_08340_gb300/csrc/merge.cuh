@@ -24,6 +24,27 @@ __device__ __forceinline__ void merge_offer32(WarpMerger<KP>& m, uint64_t key) {
   m.count += __popc(bits);
 }
 
+// Writes result o of the merge: a key's id (split into the corpus and the id
+// within it for a search over two stacked corpora) and score, or the empty
+// result (-1, -inf).
+__device__ __forceinline__ void store_result(const ListSet& ls, int64_t* out_ids, float* out_scores,
+                                             int64_t o, uint64_t key) {
+  if (key == kEmptyKey) {
+    out_ids[o] = -1;
+    out_scores[o] = -INFINITY;
+    if (ls.out_src != nullptr) ls.out_src[o] = -1;
+    return;
+  }
+  int64_t id = static_cast<int64_t>(key_id(key));
+  if (ls.out_src != nullptr) {
+    const bool second = id >= ls.split;
+    ls.out_src[o] = second ? 1 : 0;
+    if (second) id -= ls.split;
+  }
+  out_ids[o] = id;
+  out_scores[o] = key_score(key);
+}
+
 // Lists that exist for the query tile `tile` (see ListSet).
 __device__ __forceinline__ int merge_list_count(const ListSet& ls, int tile) {
   int np = ls.P;
@@ -103,8 +124,7 @@ __device__ __forceinline__ void merge_one_query(const ListSet& ls, int qi, int k
     for (int i = lane; i < k; i += 32) {
       const uint64_t key = f.sbuf[i];
       const int64_t o = static_cast<int64_t>(qi) * k + i;
-      out_ids[o] = key == kEmptyKey ? -1 : static_cast<int64_t>(key_id(key));
-      out_scores[o] = key == kEmptyKey ? -INFINITY : key_score(key);
+      store_result(ls, out_ids, out_scores, o, key);
     }
   }
   __syncthreads();

@@ -315,10 +315,11 @@ struct SearchLayout {
 size_t round256(size_t b) { return (b + 255) / 256 * 256; }
 
 SearchLayout search_layout(oprag_index* idx, int q, int k, int path, int block_n, int pair,
-                           bool lex = false) {
+                           bool lex = false, int64_t n_second = 0) {
   SearchLayout L;
   SearchShape s{idx->n, idx->d, q, k};
   s.fused_lex = lex && path == 2;
+  s.n_second = path == 2 ? n_second : 0;
   L.path = path;
   if (path == 1) {
     L.simt_grid = simt_grid(s, idx->num_sms);
@@ -353,11 +354,16 @@ SearchLayout search_layout(oprag_index* idx, int q, int k, bool lex = false) {
 
 // Enqueues the passes of a laid-out search and its merge.  scratch holds
 // L.total() bytes; qf / gen are the shared bounds (used when L.floors).
+// E2 / n2 (tensor-core path): a second corpus stacked after the index's rows
+// in the same launches; the final merge then writes out_src (0: the index,
+// 1: the second corpus) and ids within each.
 int launch_search(oprag_index* idx, const SearchLayout& L, const void* Q, int q, int k,
                   const Fusion& fu, void* scratch, uint64_t* qf, uint32_t gen, int64_t* out_ids,
-                  float* out_scores, cudaStream_t st) {
+                  float* out_scores, cudaStream_t st, const void* E2 = nullptr, int64_t n2 = 0,
+                  int32_t* out_src = nullptr) {
   SearchShape s{idx->n, idx->d, q, k};
   s.fused_lex = L.path == 2 && fu.gathered();
+  s.n_second = L.path == 2 ? n2 : 0;
   ListSet lists{};
   cudaError_t e;
   if (idx->timing) cudaEventRecord(idx->ev[1], st);
@@ -381,7 +387,7 @@ int launch_search(oprag_index* idx, const SearchLayout& L, const void* Q, int q,
       level_cnt = reinterpret_cast<int*>(levels + static_cast<size_t>(q) * kLevels);
       ListSet slists{};
       e = launch_tc_search(idx->emb, Q, s32, fu, L.splan, sbase, idx->dev_err, &slists, st,
-                           nullptr, nullptr, 0, nullptr, nullptr, idx->wait_limit);
+                           nullptr, nullptr, 0, nullptr, nullptr, idx->wait_limit, nullptr, E2);
       if (e == cudaSuccess) e = launch_merge(slists, q, k, sids, sscores, st, kth, levels);
       if (e == cudaSuccess)
         e = cudaMemsetAsync(level_cnt, 0, static_cast<size_t>(q) * kLevels * sizeof(int), st);
@@ -397,11 +403,15 @@ int launch_search(oprag_index* idx, const SearchLayout& L, const void* Q, int q,
       idx->phases_grid = L.plan.grid;
     }
     e = launch_tc_search(idx->emb, Q, s, fu, L.plan, scratch, idx->dev_err, &lists, st, floor,
-                         L.floors ? qf : nullptr, gen, levels, level_cnt, idx->wait_limit, ph);
+                         L.floors ? qf : nullptr, gen, levels, level_cnt, idx->wait_limit, ph, E2);
   }
   if (e != cudaSuccess) return cuda_fail(e, "search kernel");
   if (idx->timing) cudaEventRecord(idx->ev[2], st);
   note_launch(idx, L.path, L.plan);
+  if (out_src != nullptr) {
+    lists.split = idx->n;
+    lists.out_src = out_src;
+  }
   e = launch_merge(lists, q, k, out_ids, out_scores, st);
   if (e != cudaSuccess) return cuda_fail(e, "merge kernel");
   if (idx->timing) cudaEventRecord(idx->ev[3], st);
@@ -796,12 +806,37 @@ int oprag_search_two(oprag_index* knowledge, oprag_index* memory, const void* qu
   if (q < 0) return fail(OPRAG_ERR_INVALID_ARG, "q < 0");
   if (q == 0) return ok();
   if (!queries || !out_ids || !out_scores) return fail(OPRAG_ERR_INVALID_ARG, "NULL argument");
-  const int ka = static_cast<int>(std::min<int64_t>(k, knowledge->n));
-  const int kb = static_cast<int>(std::min<int64_t>(k, memory->n));
   DeviceGuard g(knowledge->device);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  // Each index's top-k into its own candidate buffer, then one merge.
   int rc;
+  if (choose_path(knowledge, q) == 2 && choose_path(memory, q) == 2) {
+    // One search over both (Sec. 3.6 / Sec. 4.4: the two indices searched the
+    // same way into one ranking): the memory index's corpus tiles follow the
+    // knowledge index's in the same launches, its chunks keyed after the
+    // knowledge ids, so equal scores rank knowledge first; the merge writes
+    // the source and the id within it.  Scratch and bounds of the knowledge
+    // index.
+    const SearchLayout L = search_layout(knowledge, q, k, 2, knowledge->opt_block_n,
+                                         knowledge->opt_pair, false, memory->n);
+    if ((rc = knowledge->ensure(&knowledge->scratch, &knowledge->scratch_bytes, L.total(),
+                                "search scratch")))
+      return rc;
+    uint64_t* qf = nullptr;
+    uint32_t gen = 0;
+    if (L.floors && (rc = shared_floors(knowledge, q, st, &qf, &gen))) return rc;
+    if ((rc = begin_call(knowledge, st))) return rc;
+    if ((rc = begin_call(memory, st))) return rc;
+    const Fusion none{nullptr, 0, nullptr, 0.f};
+    knowledge->timed_lex = false;
+    if ((rc = launch_search(knowledge, L, queries, q, k, none, knowledge->scratch, qf, gen, out_ids,
+                            out_scores, st, memory->emb, memory->n, out_src)))
+      return rc;
+    if ((rc = end_call(memory, st))) return rc;
+    return end_call(knowledge, st);
+  }
+  // fp32 indices (SIMT kernel): each index's top-k, then one two-list merge.
+  const int ka = static_cast<int>(std::min<int64_t>(k, knowledge->n));
+  const int kb = static_cast<int>(std::min<int64_t>(k, memory->n));
   if ((rc = knowledge->ensure(&knowledge->cand, &knowledge->cand_bytes,
                               static_cast<size_t>(q) * ka * 12, "two-index results")))
     return rc;

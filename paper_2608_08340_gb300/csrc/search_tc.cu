@@ -65,7 +65,8 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
   } else {
     // Few units (small query batches): 128-row tiles give every SM more of
     // them; the MMA rate per row is the same for N = 128 and N = 256.
-    const int64_t units256 = static_cast<int64_t>(pl.qt) * ((s.n + 255) / 256);
+    const int64_t units256 =
+      static_cast<int64_t>(pl.qt) * ((s.n + 255) / 256 + (s.n_second + 255) / 256);
     if (units256 < 4LL * num_sms) bn = 128;
   }
   // Dual mode: every unit takes two query tiles and one 128-row corpus tile,
@@ -77,7 +78,8 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
   // 1024); it needs the two epilogue sets of lists of 8 or 16.
   const bool dual_ok = !s.fused_lex && pl.qt >= 2 && epi_sets(list_len_for(s.k)) == 2 &&
                        force_pair != 2 && (force_block_n == 0 || force_block_n == 128);
-  const int64_t dual_units = static_cast<int64_t>((pl.qt + 1) / 2) * ((s.n + 127) / 128);
+  const int64_t dual_units =
+      static_cast<int64_t>((pl.qt + 1) / 2) * ((s.n + 127) / 128 + (s.n_second + 127) / 128);
   pl.dual = dual_ok && (force_pair == 3 || (force_pair == 0 && dual_units <= 4LL * num_sms));
   if (pl.dual) bn = 128;
   pl.block_n = bn;
@@ -93,7 +95,9 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
   pl.pair = pair ? 2 : 1;
   pl.uqt = pair || pl.dual ? (pl.qt + 1) / 2 : pl.qt;
   pl.tile_stride = tile_stride < 1 ? 1 : tile_stride;
-  const int64_t all_tiles = (s.n + bn - 1) / bn;
+  // two stacked corpora: the second's tiles follow the first's
+  pl.nt_first = static_cast<int>((s.n + bn - 1) / bn);
+  const int64_t all_tiles = pl.nt_first + (s.n_second + bn - 1) / bn;
   pl.nt = static_cast<int>((all_tiles + pl.tile_stride - 1) / pl.tile_stride);
   const int64_t units = static_cast<int64_t>(pl.nt) * pl.uqt;
   const int slots = pair ? pair_capacity : num_sms;     // schedule units in flight
@@ -165,7 +169,8 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
                              const TcPlan& pl, void* scratch, int* dev_err, ListSet* lists,
                              cudaStream_t st, const float* init_floor, uint64_t* qfloor,
                              uint32_t gen, const float* levels, int* level_cnt,
-                             long long wait_limit, unsigned long long* phases) {
+                             long long wait_limit, unsigned long long* phases,
+                             const void* E2) {
   TcMaps maps;
   // With a single query tile only its real rows are loaded (the remaining
   // rows of the A tile hold stale data whose TMEM lanes the epilogue never
@@ -186,6 +191,12 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
         !make_map(&maps.qb, fu.lex_qcount, s.q, kLexK, a_rows) ||
         !make_map(&maps.eb, fu.lex_wsplit, s.n, kLexK, pl.block_n))
       return cudaErrorInvalidValue;
+  } else if (s.n_second > 0) {
+    // the second stacked corpus (dense search over two indices)
+    if (E2 == nullptr || fu.bm25 != nullptr ||
+        !make_map(&maps.eb, E2, s.n_second, s.d, pl.block_n / pl.pair))
+      return cudaErrorInvalidValue;
+    maps.qb = maps.q;
   } else {
     maps.qb = maps.q;
     maps.eb = maps.e;
@@ -194,7 +205,9 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
   const int stride = K > 32 ? 2 * K : K;
   const size_t rows = list_rows(pl);
   TcParams prm{};
-  prm.n = s.n;
+  prm.n = s.n + s.n_second;
+  prm.n_first = s.n;
+  prm.nt_first = pl.nt_first;
   prm.d = s.d;
   prm.q = s.q;
   prm.k = s.k;

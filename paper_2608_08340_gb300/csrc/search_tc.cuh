@@ -57,7 +57,9 @@ constexpr uint32_t kAStageBytes = kBlockM * kBlockK * 2;
 constexpr int kSmemBudget = 200 * 1024;
 
 struct TcParams {
-  int64_t n;
+  int64_t n;            // corpus rows (of both corpora when two are stacked)
+  int64_t n_first;      // rows of the first corpus (n for one corpus)
+  int nt_first;         // corpus tiles of the first corpus (nt-unstrided; all for one)
   int d;
   int q;
   int k;
@@ -897,8 +899,14 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
   auto a_row = [&](int J) {
     return (kPair ? 2 * J + static_cast<int>(rank) : kDual ? 2 * J : J) * kBlockM;
   };
+  // Corpus tile t: tiles [0, nt_first) of the first corpus (map_e), then
+  // those of the second (map_eb) when two are stacked (dense searches only).
   auto b_row = [&](int t) {
-    return t * BN + (kPair ? static_cast<int>(rank) * (BN / 2) : 0);
+    const int tl = t < p.nt_first ? t : t - p.nt_first;
+    return tl * BN + (kPair ? static_cast<int>(rank) * (BN / 2) : 0);
+  };
+  auto b_map = [&](int t) -> const CUtensorMap* {
+    return kLex == kLexNone && t >= p.nt_first ? &map_eb : &map_e;
   };
 
   if (threadIdx.x == 0) {
@@ -915,7 +923,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     fence_mbar_init();
     prefetch_map(&map_q);
     prefetch_map(&map_e);
-    if constexpr (kHybrid) {
+    if (kHybrid || p.n_first < p.n) {
       prefetch_map(&map_qb);
       prefetch_map(&map_eb);
     }
@@ -928,7 +936,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       if (leader) mbar_arrive_expect_tx(&full[s], stage_tx);
       const uint32_t bar = cluster_addr(&full[s], 0);                  // the leader's full[s]
       tma_load_2d_pair(sA + s * kAStage, &map_q, bar, kb * kBlockK, a_row(J));
-      tma_load_2d_pair(sB + s * kBStageBytes, &map_e, bar, kb * kBlockK, b_row(t));
+      tma_load_2d_pair(sB + s * kBStageBytes, b_map(t), bar, kb * kBlockK, b_row(t));
     } else if (kHybrid && kb == p.kblocks) {
       // the head-term stage: counts x split weights (one 64-element K block)
       mbar_arrive_expect_tx(&full[s], stage_tx);
@@ -940,7 +948,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       if constexpr (kDual)
         tma_load_2d(sA + s * kAStage + kAStageBytes, &map_q, &full[s], kb * kBlockK,
                     a_row(J) + kBlockM);
-      tma_load_2d(sB + s * kBStageBytes, &map_e, &full[s], kb * kBlockK, b_row(t));
+      tma_load_2d(sB + s * kBStageBytes, b_map(t), &full[s], kb * kBlockK, b_row(t));
     }
   };
   int pre_issued = 0;           // stages the producer issued before the setup barrier
@@ -1138,6 +1146,11 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       const int J = us.j();
       const int j = qtile(J);                // this CTA's query tile
       const int64_t t = us.t();
+      // Chunk ids of this corpus tile: its rows, after the first corpus's
+      // n_first ids when it belongs to a stacked second corpus.
+      const bool second = t >= p.nt_first;
+      const int64_t id_base = second ? p.n_first + (t - p.nt_first) * BN : t * BN;
+      const int64_t id_end = second ? p.n : p.n_first;
       const bool valid = j * kBlockM + row < p.q;
       const bool warp_live = j * kBlockM + eg * 32 < p.q;
       if (J != cur_j) {
@@ -1197,11 +1210,11 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         auto scores = [&](const uint32_t (&r)[32], int c, float (&v)[32]) {
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-          const int64_t id0 = t * BN + c * 32;
+          const int64_t id0 = id_base + c * 32;
           if constexpr (kLex == kLexBlock) {
             if (act) {
               const float a = p.fu.alpha, b1 = 1.f - p.fu.alpha;
-              if (id0 + 32 <= p.n) {
+              if (id0 + 32 <= id_end) {
 #pragma unroll
                 for (int i = 0; i < 32; i += 4) {
                   const float4 w = *reinterpret_cast<const float4*>(brow + id0 + i);
@@ -1213,7 +1226,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
               } else {
 #pragma unroll
                 for (int i = 0; i < 32; ++i)
-                  if (id0 + i < p.n) v[i] = fmaf(a, v[i], b1 * (brow[id0 + i] * inv_max));
+                  if (id0 + i < id_end) v[i] = fmaf(a, v[i], b1 * (brow[id0 + i] * inv_max));
               }
             }
           }
@@ -1248,17 +1261,17 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
               }
             }
           }
-          if (id0 + 32 > p.n) {
+          if (id0 + 32 > id_end) {
 #pragma unroll
             for (int i = 0; i < 32; ++i)
-              if (id0 + i >= p.n) v[i] = -INFINITY;
+              if (id0 + i >= id_end) v[i] = -INFINITY;
           }
         };
         // Filters one chunk against max(list floor, unit bound).
         auto process = [&](const uint32_t (&r)[32], int c, float bound) {
           float v[32];
           scores(r, c, v);
-          const int64_t id0 = t * BN + c * 32;
+          const int64_t id0 = id_base + c * 32;
           list.sync(false, act);
           const float fl = fmaxf(list.floor(), bound);
           if (__any_sync(0xffffffffu, act && max32(v) >= fl)) {

@@ -103,3 +103,50 @@ def test_search_two_matches_the_stacked_oracle(nk, nm, k):
     check_dense(stacked, sc.cpu().numpy(), E, w.Q_data, k, f"two indices {nk}+{nm}")
     kn.check()
     mem.check()
+
+
+@pytest.mark.parametrize("nk,nm,q,k", [(32768, 8192, 256, 5), (9000, 300, 40, 16),
+                                       (20000, 45000, 130, 100), (256, 70000, 600, 7),
+                                       (1000, 1, 3, 2)])
+def test_search_two_is_one_search_over_the_stacked_rows(nk, nm, q, k):
+    """The two-index search runs one search pass (and, for k > 32 over many
+    tiles, one sampled pass) over the knowledge rows followed by the memory
+    rows: its results equal a search of one index holding the stacked rows,
+    with memory ids shifted by the knowledge size (scores within 1e-6, ids
+    equal outside 1e-6 near-ties: the two runs may tile the rows
+    differently); equal scores rank the knowledge index first."""
+    w = workloads.config(1, n=nk + nm, batch=q)
+    E = w.E_data
+    kn, mem = Index(dev_tensor(E[:nk])), Index(dev_tensor(E[nk:]))
+    both = Index(dev_tensor(E))
+    Q = dev_tensor(w.Q_data)
+    ids, src, sc = search_two(kn, mem, Q, k)
+    r_ids, r_sc = both.search(Q, k)
+    torch.cuda.synchronize()
+    src = src.cpu().numpy()
+    assert ((src == 0) | (src == 1)).all()
+    ids = ids.cpu().numpy()
+    assert (ids[src == 0] < nk).all() and (ids[src == 1] < nm).all()
+    stacked = np.where(src == 1, ids + nk, ids)
+    r_ids, r_sc = r_ids.cpu().numpy(), r_sc.cpu().numpy()
+    np.testing.assert_allclose(sc.cpu().numpy(), r_sc, rtol=0, atol=1e-6)
+    tie = np.zeros_like(r_sc, dtype=bool)
+    tie[:, 1:] |= (r_sc[:, :-1] - r_sc[:, 1:]) <= 1e-6
+    tie[:, :-1] |= (r_sc[:, :-1] - r_sc[:, 1:]) <= 1e-6
+    np.testing.assert_array_equal(stacked[~tie], r_ids[~tie])
+    rows = np.arange(q) if q <= 64 else np.sort(np.random.default_rng(q).choice(q, 48, replace=False))
+    check_dense(stacked, sc.cpu().numpy(), E, w.Q_data, k, f"stacked {nk}+{nm}", rows=rows)
+    kn.check()
+    mem.check()
+
+
+def test_search_two_ties_rank_knowledge_first():
+    """The same row in both indices: the knowledge copy comes first."""
+    rng = np.random.default_rng(4)
+    E = workloads.to_bf16_bits(workloads._normalise(rng.standard_normal((500, 64)).astype(np.float32)))
+    kn, mem = Index(dev_tensor(E)), Index(dev_tensor(E[::-1].copy()))
+    ids, src, sc = search_two(kn, mem, dev_tensor(E[:5]), 2)
+    torch.cuda.synchronize()
+    assert src.cpu().tolist() == [[0, 1]] * 5
+    assert ids.cpu().tolist() == [[i, 499 - i] for i in range(5)]
+    assert (sc[:, 0] == sc[:, 1]).all()
