@@ -5,6 +5,7 @@
 #include <cstddef>
 #include <cstdint>
 #include <cuda_runtime.h>
+#include <cuda_bf16.h>
 
 namespace oprag {
 
@@ -217,6 +218,33 @@ struct LexPrep {
 cudaError_t launch_lex_prep(const int32_t* lex_class, const int64_t* post_ptr, int vocab,
                             const int32_t* q_indptr, const int32_t* q_terms, int q,
                             const LexPrep& out, cudaStream_t st);
+
+// --- building the lexical index on the device (sparse_build.cu): from a
+// term-major inverted index of (chunk, tf) pairs (term_start: vocab + 1
+// offsets into inv), each chunk's token count and each term's idf, every
+// per-posting weight, written to the postings (terms with slot < 0, at
+// post_ptr[t]), the dense rows (slot >= 0), the split head-term operand
+// (lex_class >= 0) and the mid rows (lex_class <= -2); then the per-tile
+// postings table.  Destinations of dense rows, wsplit and mid_w must be
+// zeroed beforehand.
+struct LexBuild {
+  int vocab;
+  const int2* inv;
+  const int64_t* term_start;
+  const double* idf;
+  const int32_t* doc_len;
+  double avgdl, k1, b;
+  const int32_t* slot;
+  const int32_t* lex_class;
+  const int64_t* post_ptr;
+  int2* post;
+  float* dense_w;
+  int64_t dense_ld;
+  __nv_bfloat16* wsplit;
+  float* mid_w;
+  int64_t mid_ld;
+};
+cudaError_t launch_lex_build(const LexBuild& lb, int ntiles, int64_t* tile_ptr, cudaStream_t st);
 
 // --- lexical rerank of a dense top-N (dense-first hybrid), rerank.cu.
 // cand_ids / cand_scores: q x ncand dense results (id -1 = none), ncand <=

@@ -7,6 +7,7 @@
 #include <cstring>
 #include <mutex>
 #include <string>
+#include <thread>
 #include <vector>
 
 #include "oprag.h"
@@ -38,21 +39,6 @@ int ok() {
 }
 
 size_t elem_size(int dtype) { return dtype == OPRAG_F32 ? 4 : 2; }
-
-// bf16 bit pattern of a finite float, rounded to nearest even.
-uint16_t f32_to_bf16_rne(float f) {
-  uint32_t u;
-  std::memcpy(&u, &f, sizeof(u));
-  u += 0x7FFFu + ((u >> 16) & 1u);
-  return static_cast<uint16_t>(u >> 16);
-}
-
-float bf16_to_f32(uint16_t h) {
-  const uint32_t u = static_cast<uint32_t>(h) << 16;
-  float f;
-  std::memcpy(&f, &u, sizeof(f));
-  return f;
-}
 
 // Makes the index's device current for the duration of a call.
 struct DeviceGuard {
@@ -958,10 +944,14 @@ int oprag_search_host(oprag_index* idx, const void* queries, int32_t q, int32_t 
   return *idx->err_host != 0 ? oprag_index_check(idx) : ok();
 }
 
-// Builds the device side of BM25 (per-posting weights, dense rows of the
-// commonest terms, postings) from the index's host copy of the token bags,
-// in fp64 on the host.  Called whenever the bags or the chunk count change,
-// so that df, avgdl and every weight follow the current corpus.
+// Builds the device side of BM25 from the index's host copy of the token
+// bags.  Called whenever the bags or the chunk count change, so that df,
+// avgdl and every weight follow the current corpus.  The host does the
+// integer work -- a stable counting sort of the bags into a term-major
+// inverted index of (chunk, tf) pairs, chunks ascending, on several threads
+// over contiguous chunk ranges; document frequencies, lengths, idf and the
+// terms' storage classes -- and the device computes every weight from it
+// (launch_lex_build).
 int rebuild_sparse(oprag_index* idx) {
   const int64_t n = idx->n;
   const int vocab = idx->vocab;
@@ -970,27 +960,80 @@ int rebuild_sparse(oprag_index* idx) {
   const int32_t* doc_terms = idx->bag_terms.data();
   const int64_t total = doc_indptr[n];
 
-  // Term frequencies per chunk, document frequencies, average length.
-  std::vector<int64_t> df(vocab, 0);
-  std::vector<int32_t> tmp;
-  std::vector<int32_t> pair_doc, pair_term, pair_tf;
-  pair_doc.reserve(total);
-  pair_term.reserve(total);
-  pair_tf.reserve(total);
-  for (int64_t dd = 0; dd < n; ++dd) {
-    tmp.assign(doc_terms + doc_indptr[dd], doc_terms + doc_indptr[dd + 1]);
-    std::sort(tmp.begin(), tmp.end());
-    for (size_t i = 0; i < tmp.size();) {
-      size_t j = i;
-      while (j < tmp.size() && tmp[j] == tmp[i]) ++j;
-      pair_doc.push_back(static_cast<int32_t>(dd));
-      pair_term.push_back(tmp[i]);
-      pair_tf.push_back(static_cast<int32_t>(j - i));
-      df[tmp[i]] += 1;
-      i = j;
+  // Pass 1: per thread (a contiguous range of chunks), the number of chunks
+  // holding each term.  Pass 2: each thread writes its (chunk, tf) pairs at
+  // its own offsets inside each term's range, so chunks stay ascending.
+  const int T = static_cast<int>(std::max<int64_t>(
+      1, std::min<int64_t>({static_cast<int64_t>(std::thread::hardware_concurrency()), 16,
+                            (n + 1023) / 1024})));
+  std::vector<std::vector<int64_t>> cnt(T, std::vector<int64_t>(vocab, 0));
+  auto chunk_range = [&](int th, int64_t* d0, int64_t* d1) {
+    *d0 = n * th / T;
+    *d1 = n * (th + 1) / T;
+  };
+  // Per distinct term of chunk dd: f(term, tf), in first-occurrence order.
+  auto each_term = [&](int64_t dd, std::vector<int32_t>& last, std::vector<int32_t>& tfc,
+                       std::vector<int32_t>& seen, auto&& f) {
+    seen.clear();
+    for (int32_t i = doc_indptr[dd]; i < doc_indptr[dd + 1]; ++i) {
+      const int32_t t = doc_terms[i];
+      if (last[t] != static_cast<int32_t>(dd)) {
+        last[t] = static_cast<int32_t>(dd);
+        tfc[t] = 0;
+        seen.push_back(t);
+      }
+      ++tfc[t];
+    }
+    for (int32_t t : seen) f(t, tfc[t]);
+  };
+  auto run = [&](auto&& body) {
+    std::vector<std::thread> pool;
+    for (int th = 1; th < T; ++th) pool.emplace_back(body, th);
+    body(0);
+    for (auto& p : pool) p.join();
+  };
+  run([&](int th) {
+    int64_t d0, d1;
+    chunk_range(th, &d0, &d1);
+    std::vector<int32_t> last(vocab, -1), tfc(vocab, 0), seen;
+    for (int64_t dd = d0; dd < d1; ++dd)
+      each_term(dd, last, tfc, seen, [&](int32_t t, int32_t) { ++cnt[th][t]; });
+  });
+  std::vector<int64_t> df(vocab, 0), term_start(static_cast<size_t>(vocab) + 1, 0);
+  for (int t = 0; t < vocab; ++t) {
+    for (int th = 0; th < T; ++th) df[t] += cnt[th][t];
+    term_start[t + 1] = term_start[t] + df[t];
+  }
+  const int64_t nnz_all = term_start[vocab];
+  // cnt becomes each thread's write offset per term
+  for (int t = 0; t < vocab; ++t) {
+    int64_t off = term_start[t];
+    for (int th = 0; th < T; ++th) {
+      const int64_t c = cnt[th][t];
+      cnt[th][t] = off;
+      off += c;
     }
   }
+  std::vector<int2> inv(static_cast<size_t>(std::max<int64_t>(nnz_all, 1)));
+  run([&](int th) {
+    int64_t d0, d1;
+    chunk_range(th, &d0, &d1);
+    std::vector<int32_t> last(vocab, -1), tfc(vocab, 0), seen;
+    for (int64_t dd = d0; dd < d1; ++dd)
+      each_term(dd, last, tfc, seen, [&](int32_t t, int32_t tf) {
+        inv[cnt[th][t]++] = make_int2(static_cast<int32_t>(dd), tf);
+      });
+  });
+  std::vector<int32_t> doc_len(static_cast<size_t>(std::max<int64_t>(n, 1)));
+  for (int64_t dd = 0; dd < n; ++dd) doc_len[dd] = doc_indptr[dd + 1] - doc_indptr[dd];
   const double avgdl = n > 0 ? static_cast<double>(total) / static_cast<double>(n) : 0.0;
+  const double N = static_cast<double>(n);
+  std::vector<double> idf(vocab);
+  for (int t = 0; t < vocab; ++t) {
+    const double dft = static_cast<double>(df[t]);
+    idf[t] = std::log(1.0 + (N - dft + 0.5) / (dft + 0.5));
+  }
+
   // Terms in more than half of the chunks become dense rows of the BM25 pass
   // and the rerank; the others keep postings grouped by term, chunks
   // ascending inside a term.
@@ -1016,106 +1059,88 @@ int rebuild_sparse(oprag_index* idx) {
     for (int t = 0; t < vocab; ++t)
       if (df[t] >= floor_df) order.push_back(t);
     std::stable_sort(order.begin(), order.end(),
-                     [&](int32_t a, int32_t c) { return df[a] > df[c]; });
+                     [&](int32_t x, int32_t y) { return df[x] > df[y]; });
     const int64_t mid_cap = kLexMidBytes / (mld * 4);
     for (int32_t t : order) {
-      if (n_tc < kLexHeadTerms) {
-        lex_class[t] = n_tc++;
-      } else if (slot[t] >= 0 || n_mid < mid_cap) {
-        lex_class[t] = -2 - n_mid++;
-      }
+      if (n_tc < kLexHeadTerms) lex_class[t] = n_tc++;
+      else if (slot[t] >= 0 || n_mid < mid_cap) lex_class[t] = -2 - n_mid++;
     }
   }
-  std::vector<float> dense(static_cast<size_t>(n_dense) * dld, 0.f);
-  std::vector<float> mid(static_cast<size_t>(std::max(n_mid, 1)) * mld, 0.f);
-  // Head-term weights per chunk as the tensor-core operand of the gathered
-  // hybrid search: n rows of kLexK bf16, slot s's weight w rounded to nearest
-  // even (high half) at s and the rounded remainder w - high (low half) at
-  // kLexHeadTerms + s; high + low is within 2^-16 |w| of w.
-  std::vector<uint16_t> wsplit(static_cast<size_t>(n) * kLexK, 0);
   std::vector<int64_t> ptr(static_cast<size_t>(vocab) + 1, 0);
   for (int t = 0; t < vocab; ++t) ptr[t + 1] = ptr[t] + (slot[t] < 0 ? df[t] : 0);
   const int64_t nnz = ptr[vocab];
-  if (nnz >= (int64_t(1) << 31))
+  if (nnz >= (int64_t(1) << 31) || nnz_all >= (int64_t(1) << 31))
     return fail(OPRAG_ERR_INVALID_ARG, "more than 2^31 postings");
-  std::vector<int2> post(nnz);
-  std::vector<int64_t> fill(ptr.begin(), ptr.end() - 1);
-  const double N = static_cast<double>(n);
-  for (size_t i = 0; i < pair_doc.size(); ++i) {
-    const int32_t t = pair_term[i], dd = pair_doc[i];
-    const double len = static_cast<double>(doc_indptr[dd + 1] - doc_indptr[dd]);
-    const double norm = 1.0 - b + b * (avgdl > 0.0 ? len / avgdl : 0.0);
-    const double dft = static_cast<double>(df[t]);
-    const double idf = std::log(1.0 + (N - dft + 0.5) / (dft + 0.5));
-    const double tf = static_cast<double>(pair_tf[i]);
-    const float wt = static_cast<float>(idf * tf * (k1 + 1.0) / (tf + k1 * norm));
-    if (slot[t] >= 0) {
-      dense[static_cast<size_t>(slot[t]) * dld + dd] = wt;
-    } else {
-      int32_t bits;
-      std::memcpy(&bits, &wt, sizeof(bits));
-      post[fill[t]++] = make_int2(dd, bits);
-    }
-    const int c = lex_class[t];
-    if (c >= 0) {
-      const uint16_t hi = f32_to_bf16_rne(wt);
-      wsplit[static_cast<size_t>(dd) * kLexK + c] = hi;
-      wsplit[static_cast<size_t>(dd) * kLexK + kLexHeadTerms + c] =
-          f32_to_bf16_rne(wt - bf16_to_f32(hi));
-    } else if (c <= -2) {
-      mid[static_cast<size_t>(-2 - c) * mld + dd] = wt;
-    }
-  }
-  // Where each term's postings enter each tile of the BM25 pass.
   const int ntiles = static_cast<int>((n + kBm25DocTile - 1) / kBm25DocTile);
-  std::vector<int64_t> tptr(static_cast<size_t>(vocab) * (ntiles + 1));
-  for (int t = 0; t < vocab; ++t) {
-    int64_t* row = tptr.data() + static_cast<size_t>(t) * (ntiles + 1);
-    int64_t p = ptr[t];
-    for (int tb = 0; tb <= ntiles; ++tb) {
-      const int64_t doc0 = static_cast<int64_t>(tb) * kBm25DocTile;
-      while (p < ptr[t + 1] && post[p].x < doc0) ++p;
-      row[tb] = p;
-    }
-  }
 
   DeviceGuard g(idx->device);
   cudaError_t e = idx->drain();
   if (e != cudaSuccess) return cuda_fail(e, "waiting for pending work");
   idx->free_sparse();
   idx->has_sparse = false;
+  const size_t dense_elems = std::max<size_t>(static_cast<size_t>(n_dense) * dld, 4);
+  const size_t wsplit_elems = static_cast<size_t>(n) * kLexK;
+  const size_t mid_elems = static_cast<size_t>(std::max(n_mid, 1)) * mld;
+  const size_t tptr_elems = static_cast<size_t>(vocab) * (ntiles + 1);
+  // temporaries of the build: the inverted index, term offsets, idf, lengths
+  int2* d_inv = nullptr;
+  int64_t* d_start = nullptr;
+  double* d_idf = nullptr;
+  int32_t* d_len = nullptr;
+  auto free_tmp = [&]() {
+    if (d_inv) cudaFree(d_inv);
+    if (d_start) cudaFree(d_start);
+    if (d_idf) cudaFree(d_idf);
+    if (d_len) cudaFree(d_len);
+  };
   if (cudaMalloc(&idx->post_ptr, ptr.size() * sizeof(int64_t)) != cudaSuccess ||
       cudaMalloc(&idx->post, std::max<int64_t>(nnz, 1) * sizeof(int2)) != cudaSuccess ||
       cudaMalloc(&idx->dense_slot, slot.size() * sizeof(int32_t)) != cudaSuccess ||
-      cudaMalloc(&idx->dense_w, std::max<size_t>(dense.size(), 4) * sizeof(float)) != cudaSuccess ||
-      cudaMalloc(&idx->tile_ptr, tptr.size() * sizeof(int64_t)) != cudaSuccess ||
-      cudaMalloc(&idx->wsplit, wsplit.size() * sizeof(uint16_t)) != cudaSuccess ||
+      cudaMalloc(&idx->dense_w, dense_elems * sizeof(float)) != cudaSuccess ||
+      cudaMalloc(&idx->tile_ptr, tptr_elems * sizeof(int64_t)) != cudaSuccess ||
+      cudaMalloc(&idx->wsplit, wsplit_elems * sizeof(uint16_t)) != cudaSuccess ||
       cudaMalloc(&idx->lex_class, lex_class.size() * sizeof(int32_t)) != cudaSuccess ||
-      cudaMalloc(&idx->mid_w, mid.size() * sizeof(float)) != cudaSuccess) {
+      cudaMalloc(&idx->mid_w, mid_elems * sizeof(float)) != cudaSuccess ||
+      cudaMalloc(&d_inv, inv.size() * sizeof(int2)) != cudaSuccess ||
+      cudaMalloc(&d_start, term_start.size() * sizeof(int64_t)) != cudaSuccess ||
+      cudaMalloc(&d_idf, idf.size() * sizeof(double)) != cudaSuccess ||
+      cudaMalloc(&d_len, doc_len.size() * sizeof(int32_t)) != cudaSuccess) {
     cudaGetLastError();
+    free_tmp();
     idx->free_sparse();
     return fail(OPRAG_ERR_OOM, "cannot allocate postings");
   }
   e = cudaMemcpy(idx->post_ptr, ptr.data(), ptr.size() * sizeof(int64_t), cudaMemcpyHostToDevice);
-  if (e == cudaSuccess && nnz)
-    e = cudaMemcpy(idx->post, post.data(), nnz * sizeof(int2), cudaMemcpyHostToDevice);
   if (e == cudaSuccess)
     e = cudaMemcpy(idx->dense_slot, slot.data(), slot.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
-  if (e == cudaSuccess && !dense.empty())
-    e = cudaMemcpy(idx->dense_w, dense.data(), dense.size() * sizeof(float), cudaMemcpyHostToDevice);
-  if (e == cudaSuccess)
-    e = cudaMemcpy(idx->tile_ptr, tptr.data(), tptr.size() * sizeof(int64_t), cudaMemcpyHostToDevice);
-  if (e == cudaSuccess)
-    e = cudaMemcpy(idx->wsplit, wsplit.data(), wsplit.size() * sizeof(uint16_t),
-                   cudaMemcpyHostToDevice);
   if (e == cudaSuccess)
     e = cudaMemcpy(idx->lex_class, lex_class.data(), lex_class.size() * sizeof(int32_t),
                    cudaMemcpyHostToDevice);
   if (e == cudaSuccess)
-    e = cudaMemcpy(idx->mid_w, mid.data(), mid.size() * sizeof(float), cudaMemcpyHostToDevice);
+    e = cudaMemcpy(d_inv, inv.data(), inv.size() * sizeof(int2), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(d_start, term_start.data(), term_start.size() * sizeof(int64_t),
+                   cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(d_idf, idf.data(), idf.size() * sizeof(double), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(d_len, doc_len.data(), doc_len.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemset(idx->dense_w, 0, dense_elems * sizeof(float));
+  if (e == cudaSuccess) e = cudaMemset(idx->wsplit, 0, wsplit_elems * sizeof(uint16_t));
+  if (e == cudaSuccess) e = cudaMemset(idx->mid_w, 0, mid_elems * sizeof(float));
+  if (e == cudaSuccess) {
+    const LexBuild lb{vocab,        d_inv,           d_start,     d_idf,
+                      d_len,        avgdl,           k1,          b,
+                      idx->dense_slot, idx->lex_class, idx->post_ptr, idx->post,
+                      idx->dense_w, dld,
+                      reinterpret_cast<__nv_bfloat16*>(idx->wsplit), idx->mid_w, mld};
+    e = launch_lex_build(lb, ntiles, idx->tile_ptr, nullptr);
+  }
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  free_tmp();
   if (e != cudaSuccess) {
     idx->free_sparse();
-    return cuda_fail(e, "uploading postings");
+    return cuda_fail(e, "building the lexical index");
   }
   idx->nnz = nnz;
   idx->dense_ld = dld;
