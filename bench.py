@@ -485,6 +485,20 @@ def measure(args, cfg: int, batch: int, rank: int, world: int, local_rank: int,
 
     phases = phase_breakdown(idx, step, flush, min(args.steps, 20)) if args.phases else None
 
+    # What two CUDA events with nothing between them read after the same
+    # flush: part of every event-timed kernel duration that is not the
+    # kernel's work (reported beside the kernel time, not subtracted).
+    ev_pair = []
+    for _ in range(20):
+        flush.zero_()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        b.record(stream)
+        ev_pair.append((a, b))
+    torch.cuda.synchronize()
+    ev_pair_us = statistics.median(a.elapsed_time(b) for a, b in ev_pair) * 1e3
+
     # Warm-L2 figure, reported beside the flushed one: the same steps back to
     # back with no flush in between (a corpus under 129 MB stays in L2).
     warm_marks = []
@@ -589,6 +603,7 @@ def measure(args, cfg: int, batch: int, rank: int, world: int, local_rank: int,
     roof["kernel"] = "tc_search_kernel" if path == "tc" else "simt_search_kernel"
     roof["kernel_ms_mean"] = statistics.mean(tim["search_ms"])
     roof["kernel_ms_median"] = statistics.median(tim["search_ms"])
+    roof["event_pair_us"] = ev_pair_us
     roof["merge_ms_mean"] = statistics.mean(tim["merge_ms"])
     if sampled:
         # k > 32: the first pass over every 32nd corpus tile and its merge,
