@@ -605,10 +605,13 @@ def measure(args, cfg: int, batch: int, rank: int, world: int, local_rank: int,
     roof["kernel_ms_median"] = statistics.median(tim["search_ms"])
     roof["event_pair_us"] = ev_pair_us
     roof["merge_ms_mean"] = statistics.mean(tim["merge_ms"])
+    roof["merge_ms_median"] = statistics.median(tim["merge_ms"])
     if sampled:
         # k > 32: the first pass over every 32nd corpus tile and its merge,
         # timed apart from the main pass (the dominant kernel above)
         roof["sample_pass_ms_mean"] = statistics.mean(tim["sample_ms"])
+        roof["sample_pass_ms_median"] = statistics.median(tim["sample_ms"])
+        roof["sample_pass_ms_max"] = max(tim["sample_ms"])
     if cfg == 3 and not dense_first:
         roof["bm25_ms_mean"] = statistics.mean(tim["lexical_ms"])
         roof["sparse"] = sparse_terms(w)
