@@ -268,7 +268,9 @@ struct WarpMerger {
     k = k_;
   }
 
-  __device__ void compact() {
+  // Not inlined: the merges offer keys from unrolled loops, and one copy of
+  // the sort per offer made their code outgrow the instruction cache.
+  __device__ __noinline__ void compact() {
     const int lane = threadIdx.x & 31;
     __syncwarp();
     uint64_t v[kE];

@@ -19,7 +19,8 @@ inline int list_len_for(int k) {
 
 // Partial top-K lists written by a search kernel and read by the merge.  The
 // list of query row `row` of query tile `tile` produced by producer `p` starts
-// at keys + ((tile * P + p) * TH + row) * stride and is sorted best first.
+// at keys + ((tile * P + p) * TH + row) * stride and is sorted best first,
+// unless `counts` is set (see there).
 struct ListSet {
   const uint64_t* keys;
   int P;
@@ -39,6 +40,16 @@ struct ListSet {
   // the id and 0; -1 for an empty result).  out_src == nullptr: ids as kept.
   int64_t split = 0;
   int32_t* out_src = nullptr;
+  // Buffered tensor-core lists (k > 32) are left as the search filled them:
+  // list r (the index above without the stride) holds counts[r] <= stride
+  // keys in no order.  nullptr: sorted lists of klen keys.
+  const int* counts = nullptr;
+  // With counts: the main pass's counted floors per query (kLevels each,
+  // with one counter per band, see TcParams::levels).  A level whose band
+  // counts up to it sum to k is a proven lower bound of the query's k-th
+  // best score, so the merge drops keys below it.
+  const float* levels = nullptr;
+  const int* level_cnt = nullptr;
 };
 
 // Optional lexical part of the fused score (Sec. 4.4 weighted fusion):
@@ -139,8 +150,8 @@ size_t tc_scratch_bytes(const SearchShape& s, const TcPlan& p);
 // bounds shared by all lists, valid for entries tagged with gen (see
 // search_tc.cuh); zero-filled memory is a valid initial state.
 // levels / level_cnt (optional, q x kLevels, buffered lists only): candidate
-// floors and zeroed counters; a floor becomes a shared bound once k pushed
-// keys reach it.
+// floors (non-increasing) and zeroed counters, one per band between floors;
+// a floor becomes a shared bound once k pushed keys reach it.
 // wait_limit: cycles an mbarrier wait may spin before the kernel gives up and
 // sets *dev_err (<= 0: the default of about a second).
 // phases (optional, grid x kTcPhases zeroed words): global-timer stamps of

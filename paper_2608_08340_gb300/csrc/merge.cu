@@ -4,10 +4,11 @@
 // local candidates to the global top-k, done inside one GPU: the producers
 // are corpus slices instead of index shards.
 //
-// Three merges by list count and k: one warp per query over at most 32
-// sorted lists (head by head), one to four warps per query over up to 512
-// lists when k <= 16 (also head by head), and the block merge of merge.cuh
-// (one CTA per query) otherwise.
+// Four merges: for sorted lists, by list count and k, one warp per query
+// over at most 32 lists (head by head), one to four warps per query over up
+// to 512 lists when k <= 16 (also head by head), and the block merge of
+// merge.cuh (one CTA per query) otherwise; for unsorted lists (buffered
+// tensor-core lists, k > 32) one warp per query over all their keys.
 #include "merge.cuh"
 
 namespace oprag {
@@ -209,6 +210,120 @@ merge_small_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
   }
 }
 
+// Unsorted lists (ListSet::counts), k > 32: one warp per query.  The warp
+// scans the query's list counts into offsets in shared memory, reads the
+// concatenated keys 32 x kUnsortedLoads at a time (each key finds its list
+// by binary search over the offsets), drops keys below the counted floor and
+// keeps the rest in a WarpMerger, whose buffer is sorted only when it fills
+// up and once at the end.  A good floor leaves a few hundred keys of the
+// several thousand read, so a query usually costs one sort; the warps of
+// different queries share nothing and need no barrier.
+constexpr int kUnsortedWarps = 4;
+constexpr int kUnsortedLoads = 8;
+
+// Shared memory of merge_unsorted_kernel: a merger buffer and P + 1
+// offsets per warp.
+template <int KP>
+size_t unsorted_smem_bytes(int P) {
+  return kUnsortedWarps * (2 * KP * sizeof(uint64_t) + (static_cast<size_t>(P) + 4) / 4 * 16);
+}
+
+template <int KP>
+__global__ void __launch_bounds__(kUnsortedWarps * 32)
+merge_unsorted_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
+                      float* __restrict__ out_scores, float* __restrict__ kth_out,
+                      float* __restrict__ levels_out) {
+  extern __shared__ __align__(16) uint64_t smem_u[];
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  constexpr int kCap = 2 * KP;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int qi = blockIdx.x * kUnsortedWarps + warp;
+  if (qi >= q) return;
+  const int tile = qi / ls.TH, row = qi % ls.TH;
+  const int np = merge_list_count(ls, tile);
+  const int offs_len = (ls.P + 4) / 4 * 4;
+  int* offs = reinterpret_cast<int*>(smem_u + kUnsortedWarps * kCap) + warp * offs_len;
+  const int* cnt = ls.counts + static_cast<int64_t>(tile) * ls.P * ls.TH + row;
+  const uint64_t* base = ls.keys + (static_cast<int64_t>(tile) * ls.P * ls.TH + row) * ls.stride;
+  const int64_t list_step = static_cast<int64_t>(ls.TH) * ls.stride;
+
+  // offs[p]: keys of the lists before p (exclusive scan, 32 lists a round)
+  int total = 0;
+  for (int p0 = 0; p0 < np; p0 += 32) {
+    const int p = p0 + lane;
+    const int c = p < np ? max(0, min(cnt[static_cast<int64_t>(p) * ls.TH], ls.stride)) : 0;
+    int incl = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += t;
+    }
+    if (p < np) offs[p] = total + incl - c;
+    total += __shfl_sync(0xffffffffu, incl, 31);
+  }
+  __syncwarp();
+
+  WarpMerger<KP> m;
+  m.init(smem_u + warp * kCap, k);
+  m.worst = merge_floor_key(ls, qi, k);
+  for (int g = 0; g < total; g += 32 * kUnsortedLoads) {
+    uint64_t key[kUnsortedLoads];
+#pragma unroll
+    for (int u = 0; u < kUnsortedLoads; ++u) {
+      const int i = g + u * 32 + lane;
+      key[u] = kEmptyKey;
+      if (i < total) {
+        // the last list p with offs[p] <= i (it holds key i - offs[p])
+        int p0 = 0, p1 = np - 1;
+        while (p0 < p1) {
+          const int mid = (p0 + p1 + 1) >> 1;
+          if (offs[mid] <= i) p0 = mid; else p1 = mid - 1;
+        }
+        key[u] = base[p0 * list_step + (i - offs[p0])];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kUnsortedLoads; ++u)
+      if (g + u * 32 < total) merge_offer32(m, key[u]);
+  }
+  m.finish();
+  if (kth_out != nullptr && lane == 0) {
+    const uint64_t kk = m.sbuf[k - 1];
+    kth_out[qi] = kk == kEmptyKey ? -INFINITY : key_score(kk);
+  }
+  if (levels_out != nullptr && lane < kLevels) {
+    const uint64_t kk = m.sbuf[level_rank(k, lane) - 1];
+    levels_out[static_cast<int64_t>(qi) * kLevels + lane] =
+        kk == kEmptyKey ? -INFINITY : key_score(kk);
+  }
+  for (int i = lane; i < k; i += 32)
+    store_result(ls, out_ids, out_scores, static_cast<int64_t>(qi) * k + i, m.sbuf[i]);
+}
+
+template <int KP>
+cudaError_t launch_unsorted_kp(const ListSet& ls, int q, int k, int64_t* ids, float* scores,
+                               cudaStream_t st, float* kth_out, float* levels_out) {
+  const size_t smem = unsorted_smem_bytes<KP>(ls.P);
+  if (smem > 48 * 1024) {
+    const cudaError_t e =
+        cudaFuncSetAttribute(merge_unsorted_kernel<KP>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+  }
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3((q + kUnsortedWarps - 1) / kUnsortedWarps);
+  cfg.blockDim = dim3(kUnsortedWarps * 32);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, merge_unsorted_kernel<KP>, ls, q, k, ids, scores, kth_out,
+                            levels_out);
+}
+
 template <typename Kern>
 cudaError_t launch_warp_per_query(Kern kern, int warps, const ListSet& ls, int q, int k,
                                   int64_t* out_ids, float* out_scores, cudaStream_t st,
@@ -316,6 +431,12 @@ cudaError_t launch_merge_two(int q, const int64_t* a_ids, const float* a_sc, int
 cudaError_t launch_merge(const ListSet& ls, int q, int k, int64_t* out_ids, float* out_scores,
                          cudaStream_t st, float* kth_out, float* levels_out) {
   if (q <= 0) return cudaSuccess;
+  if (ls.counts != nullptr) {
+    if (k <= 64) return launch_unsorted_kp<64>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
+    if (k <= 128)
+      return launch_unsorted_kp<128>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
+    return launch_unsorted_kp<256>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
+  }
   if (ls.P <= 32)
     return launch_warp_per_query(merge_kway_kernel, kWayWarps, ls, q, k, out_ids, out_scores, st,
                                  kth_out, levels_out);

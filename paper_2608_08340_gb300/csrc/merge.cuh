@@ -56,6 +56,26 @@ __device__ __forceinline__ int merge_list_count(const ListSet& ls, int tile) {
   return np;
 }
 
+// The smallest key that can still be among the query's k best: a counted
+// floor f whose band counts up to it sum to k or more proves k real scores
+// >= f, so every key of the top k has a score >= f (the key of score f with
+// the largest id ranks below all of them).  kEmptyKey (admit all) without
+// counted floors.
+__device__ __forceinline__ uint64_t merge_floor_key(const ListSet& ls, int qi, int k) {
+  if (ls.levels == nullptr || ls.level_cnt == nullptr) return kEmptyKey;
+  int sum = 0;
+#pragma unroll
+  for (int i = 0; i < kLevels; ++i) {
+    const int64_t o = static_cast<int64_t>(qi) * kLevels + i;
+    sum += ls.level_cnt[o];
+    if (sum >= k) {
+      const float f = ls.levels[o];
+      return f > -INFINITY ? make_key(f, kNoId) : kEmptyKey;
+    }
+  }
+  return kEmptyKey;
+}
+
 // Shared memory: (nw + 1) * 2 * KP keys.  All threads of the CTA call this;
 // it ends with a barrier, so the buffer can be reused.
 template <int KP>

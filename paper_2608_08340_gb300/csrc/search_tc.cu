@@ -240,6 +240,11 @@ cudaError_t launch_tc_search(const void* E, const void* Q, const SearchShape& s,
   lists->sets = pl.dual ? 1 : epi_sets(K, hybrid);
   lists->klen = K;
   lists->pair = pl.dual ? 2 : pl.pair;
+  if (K > 32) {
+    lists->counts = prm.meta_count;
+    lists->levels = prm.levels;
+    lists->level_cnt = prm.level_cnt;
+  }
   if (hybrid) return launch_bn128_gather(maps, prm, pl.grid, st);
   if (pl.dual) {
     if (pl.block_n != 128) return cudaErrorInvalidValue;

@@ -85,8 +85,10 @@ struct TcParams {
   uint64_t* qfloor;
   uint32_t gen;
   // Optional (buffered lists): per query, kLevels candidate floors (best
-  // first) and counters of pushed keys reaching each; a floor whose counter
-  // reached k bounds the query's k-th best score for every list.
+  // first, non-increasing) and one counter per band: counter i counts pushed
+  // keys whose best reached floor is floor i.  Counters 0..i summed count the
+  // pushed keys >= floor i; once that sum reaches k, floor i bounds the
+  // query's k-th best score for every list.
   const float* levels;
   int* level_cnt;
   // Optional (measurement): kPhases global-timer stamps per CTA (PhaseMark).
@@ -547,7 +549,7 @@ struct EpiList<K, false> {
   // The k-th best score held, for the k the list was set up with.
   __device__ __forceinline__ float kth(int) const { return t.floor; }
   __device__ __forceinline__ void sync(bool, bool) {}
-  __device__ __forceinline__ void finalize(const TcParams&, int64_t, bool) {}
+  __device__ __forceinline__ void read_ahead() {}
 };
 
 template <int K>
@@ -557,19 +559,40 @@ struct EpiList<K, true> {
   // Counted floors of the current query (see TcParams::levels).
   float lvl[kLevels];
   int* cnt;
+  // Their counts as read one unit earlier.  Counts only grow, so an older
+  // reading still proves its floors, and reading ahead keeps the L2 latency
+  // off the epilogue's path (it runs once per unit).
+  int4 seen;
   __device__ __forceinline__ void set_query(const TcParams& p, int64_t q_index, bool valid) {
     cnt = valid && p.levels != nullptr ? p.level_cnt + q_index * kLevels : nullptr;
 #pragma unroll
     for (int i = 0; i < kLevels; ++i) lvl[i] = cnt != nullptr ? p.levels[q_index * kLevels + i] : INFINITY;
+    seen = cnt != nullptr ? __ldcg(reinterpret_cast<const int4*>(cnt)) : make_int4(0, 0, 0, 0);
+    proven = kLevels;
   }
-  // The best counted floor that k pushed keys already reach (-inf if none).
-  __device__ __forceinline__ float proven_floor(int k) const {
+  // Reads the counts for the next unit of the same query.
+  __device__ __forceinline__ void read_ahead() {
+    if (cnt != nullptr) seen = __ldcg(reinterpret_cast<const int4*>(cnt));
+  }
+  // Index of the best floor proven by the last reading (kLevels: none).
+  int proven;
+  // The best counted floor that k pushed keys reached by the last reading
+  // (-inf if none); also sets `proven`.
+  __device__ __forceinline__ float proven_floor(int k) {
+    proven = kLevels;
     if (cnt == nullptr) return -INFINITY;
-    const int4 c = __ldcg(reinterpret_cast<const int4*>(cnt));
+    const int4 c = seen;
     const int cs[kLevels] = {c.x, c.y, c.z, c.w};
     float f = -INFINITY;
+    int sum = 0;
 #pragma unroll
-    for (int i = kLevels - 1; i >= 0; --i) f = cs[i] >= k ? lvl[i] : f;
+    for (int i = 0; i < kLevels; ++i) {
+      sum += cs[i];
+      if (sum >= k && proven == kLevels) {
+        proven = i;
+        f = lvl[i];
+      }
+    }
     return f;
   }
   __device__ __forceinline__ void init_mem(const TcParams& p, int64_t sr, int qidx) {
@@ -596,32 +619,36 @@ struct EpiList<K, true> {
     t.worst = kEmptyKey;
     t.floor = -INFINITY;
     cnt = nullptr;
+    proven = kLevels;
   }
   __device__ __forceinline__ bool full() const { return t.worst != kEmptyKey; }
   __device__ __forceinline__ float floor() const { return t.floor; }
   __device__ __forceinline__ void push(float s, uint32_t id) { t.push(s, id); }
-  // Pushes a candidate; a pushed key that reaches a counted floor counts
-  // towards it (fire-and-forget adds).  k counts prove k real keys >= that
-  // floor, which then bounds the query's k-th best for every list; a pushed
-  // key leaves its list only when the list holds K >= k better keys, so the
-  // proof stays valid.
+  // Pushes a candidate; a pushed key counts once, in the band of the best
+  // floor it reaches (a fire-and-forget add).  Sums of k counts prove k real
+  // keys >= a floor, which then bounds the query's k-th best for every list;
+  // a pushed key leaves its list only when the list holds K >= k better
+  // keys, so the proof stays valid.  A key whose band is at or below the
+  // best proven floor (`proven`) can prove nothing new and is not counted
+  // (counts stay lower bounds).
   __device__ __forceinline__ void insert(float s, uint32_t id) {
     if (!(s > -INFINITY)) return;
     const uint64_t key = make_key(s, id);
     if (key <= t.worst) return;
     t.buf[t.count++] = key;
     if (cnt != nullptr) {
+      int band = kLevels;
 #pragma unroll
-      for (int i = 0; i < kLevels; ++i)
-        if (s >= lvl[i]) atomicAdd(cnt + i, 1);
+      for (int i = kLevels - 1; i >= 0; --i)
+        if (s >= lvl[i]) band = i;
+      if (band < proven) atomicAdd(cnt + band, 1);
     }
   }
   __device__ __forceinline__ void sync(bool final, bool active) { t.sync(final, active); }
-  // Warp-collective: sorts the lane's buffer, best K first.
-  __device__ __forceinline__ void finalize(const TcParams& p, int64_t sr, bool valid) {
-    if (valid) load(p, sr); else clear();
-    t.sync(true, valid);
-  }
+  // No final sort: a list ends as its count and that many keys in no order
+  // (they include its best K), and the merge reads it so.  Sorting 32 lanes'
+  // buffers one after another at the end of the kernel, where nothing
+  // overlaps it, cost more than the merge's extra reads.
 };
 
 // ----------------------------------------------------------- lexical gather
@@ -1189,6 +1216,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                                  p.wait_limit);
       if (!__all_sync(0xffffffffu, got)) break;
       tc_fence_after();
+      if constexpr (K > 32) list.read_ahead();
       if (warp_live) {
         float inv_max = 0.f;
         const float* brow = nullptr;
@@ -1408,10 +1436,6 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       acc_ph ^= 1u << acc;
     }
     if (cur_j >= 0 && cur_valid) list.save(p, cur_sr);
-    if (K > 32) {
-      for (int J = 0; J < p.qt; ++J)
-        if (owns(J)) list.finalize(p, list_row(J), qtile(J) * kBlockM + row < p.q);
-    }
     // The set's last warp to finish (the slots start at zero).
     if (p.phases != nullptr && lane == 0)
       atomicMax(p.phases + static_cast<size_t>(blockIdx.x) * kPhases + kPhEpi0Done + set,

@@ -232,6 +232,34 @@ def test_large_k_with_sampled_floor(k):
     idx.check()
 
 
+def test_large_k_exact_ties_at_kth():
+    """k = 100 over 1500 distinct rows, each stored 30 times (45000 rows, so
+    the sampled first pass and the counted floors run): the 100th result
+    falls inside a group of 30 equal scores, and the merge, which drops keys
+    below the proven floor, must still return the group's lowest ids."""
+    rng = np.random.default_rng(0)
+    m, reps, d = 1500, 30, 128
+    base = oracle.round_bf16(workloads._normalise(rng.standard_normal((m, d)).astype(np.float32)))
+    E = np.ascontiguousarray(np.tile(base, (reps, 1)))
+    qrows = [3, 777, 1400]
+    Q = np.ascontiguousarray(base[qrows])
+    Bf = oracle.bf16_to_f32(base).astype(np.float64)
+    for r in qrows:       # distinct rows' scores are far apart, so only ties are ambiguous
+        s = np.sort(Bf @ Bf[r])[::-1]
+        assert (-np.diff(s[:6])).min() > 10 * TOL
+    o_ids, _ = oracle.search(E, Q, 100)
+    idx = _index(E)
+    ids, sc = idx.search(dev_tensor(Q), 100)
+    assert idx.last_path == "tc"
+    ids, sc = ids.cpu().numpy(), sc.cpu().numpy()
+    np.testing.assert_array_equal(ids, o_ids)
+    for i in range(len(qrows)):
+        grp = ids[i] % m
+        for g in np.unique(grp):
+            assert len(set(sc[i][grp == g].tolist())) == 1     # copies score alike
+    idx.check()
+
+
 def test_shared_bound_tags_wrap_around():
     """Searches share per-query k-th score bounds tagged with a 32-bit
     generation; when the tag wraps, the bounds array is cleared.  Results
