@@ -76,7 +76,7 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
   // CTA (small batches, where the copies into the SMs, not the MMAs, bound
   // the kernel; measured on 32768 x 768: faster up to 512 queries, slower at
   // 1024); it needs the two epilogue sets of lists of 8 or 16.
-  const bool dual_ok = !s.fused_lex && pl.qt >= 2 && epi_sets(list_len_for(s.k)) == 2 &&
+  const bool dual_ok = !s.fused_lex && pl.qt >= 2 && list_len_for(s.k) <= 16 &&
                        force_pair != 2 && (force_block_n == 0 || force_block_n == 128);
   const int64_t dual_units =
       static_cast<int64_t>((pl.qt + 1) / 2) * ((s.n + 127) / 128 + (s.n_second + 127) / 128);

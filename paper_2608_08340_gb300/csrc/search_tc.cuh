@@ -41,14 +41,17 @@ constexpr int kBlockM = 128;
 constexpr int kBlockK = 64;                 // bf16 per 128-byte row
 constexpr int kUmmaK = 16;
 // Epilogue warp sets: two (one per accumulator, 320 threads) for register
-// lists up to 16 keys; one set (192 threads) for the longer lists.  Ten warps
-// put three on two of the SM's four schedulers, which caps a thread at 168
-// registers; with six warps it may use 255 (measured: buffered lists with two
-// sets spill and run 11% slower).
+// lists up to 16 keys and for buffered lists; one set (192 threads) for lists
+// of 32.  Ten warps put three on two of the SM's four schedulers, which caps
+// a thread at 168 registers; with six warps it may use 255.  Buffered lists
+// fit the cap because their epilogue waits for each TMEM load before
+// filtering (no registers in flight across the filter); with two sets each
+// set has two units' time per unit.  Measured on GB300, 1M x 768 with 2048
+// queries and k = 100: main pass 2026 instead of 2060 us.
 // The gathered hybrid search keeps one set (its postings cursors advance
 // through consecutive units).
 __host__ __device__ constexpr int epi_sets(int K, bool lex = false) {
-  return K <= 16 && !lex ? 2 : 1;
+  return (K <= 16 || K > 32) && !lex ? 2 : 1;
 }
 __host__ __device__ constexpr int threads_for(int K, bool lex = false) {
   return 64 + 128 * epi_sets(K, lex);
@@ -1215,6 +1218,19 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       const bool got = mbar_wait(&tfull[acc], (acc_ph >> acc) & 1u, abort_flag, p.dev_err,
                                  p.wait_limit);
       if (!__all_sync(0xffffffffu, got)) break;
+      // Hands the accumulator back once this warp's TMEM loads of the unit
+      // are done.  Pair mode: the epilogue warps of both CTAs release it at
+      // the leader.
+      bool released = false;
+      auto release_acc = [&]() {
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          if constexpr (kPair) mbar_arrive_cluster(cluster_addr(&tempty[acc], 0));
+          else mbar_arrive(&tempty[acc]);
+        }
+        released = true;
+      };
       tc_fence_after();
       if constexpr (K > 32) list.read_ahead();
       if (warp_live) {
@@ -1300,9 +1316,11 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
           float v[32];
           scores(r, c, v);
           const int64_t id0 = id_base + c * 32;
-          list.sync(false, act);
-          const float fl = fmaxf(list.floor(), bound);
-          if (__any_sync(0xffffffffu, act && max32(v) >= fl)) {
+          if (__any_sync(0xffffffffu, act && max32(v) >= fmaxf(list.floor(), bound))) {
+            // Room for this chunk's keys in a buffered list (a compaction
+            // raises the list's floor, so the floor is read after it).
+            list.sync(false, act);
+            const float fl = fmaxf(list.floor(), bound);
             // Lanes insert their candidates together, one column per round,
             // so the warp runs max-per-lane rounds instead of the sum.
             uint32_t mask = 0;
@@ -1406,6 +1424,17 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         }
         const float lb = fmaxf(bound, gfl);     // admission bound of this unit
         __syncwarp();
+        if constexpr (K > 32) {
+          // Buffered lists: one chunk at a time, each load waited for before
+          // the filter (see epi_sets).
+#pragma unroll 1
+          for (int c = 0; c < NC; ++c) {
+            tmem_ld32_async(taddr + c * 32, ra);
+            tmem_wait_ld(ra);
+            process(ra, c, lb);
+          }
+        } else {
+        // Register lists: the next chunk's load flies while one is filtered.
         tmem_ld32_async(taddr, ra);
 #pragma unroll 1
         for (int c = 0; c < NC; c += 2) {
@@ -1414,7 +1443,16 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
           process(ra, c, lb);
           tmem_wait_ld(rb);
           if (c + 2 < NC) tmem_ld32_async(taddr + (c + 2) * 32, ra);
+          // The unit's last TMEM load has landed: hand the accumulator back
+          // to the MMA before filtering the last chunk (the gathered hybrid
+          // form still reads its second accumulator while filtering).  Only
+          // for register lists: measured on GB300, 32768 x 1024 with 4096
+          // queries and k = 10 took 217.6 instead of 218.9 us a step, while
+          // 1M x 768 with 2048 queries and k = 100 (buffered lists, one
+          // epilogue set) took 2095 instead of 2081 us in the main pass.
+          if (!kHybrid && K <= 32 && c + 2 >= NC) release_acc();
           process(rb, c + 1, lb);
+        }
         }
         if constexpr (K <= 32) {
           // Publish what this list now proves about the query's k-th best.
@@ -1425,14 +1463,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
           }
         }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) {
-        // Pair mode: the epilogue warps of both CTAs release the accumulator
-        // at the leader.
-        if constexpr (kPair) mbar_arrive_cluster(cluster_addr(&tempty[acc], 0));
-        else mbar_arrive(&tempty[acc]);
-      }
+      if (!released) release_acc();
       acc_ph ^= 1u << acc;
     }
     if (cur_j >= 0 && cur_valid) list.save(p, cur_sr);
