@@ -4,11 +4,12 @@
 // local candidates to the global top-k, done inside one GPU: the producers
 // are corpus slices instead of index shards.
 //
-// Four merges: for sorted lists, by list count and k, one warp per query
-// over at most 32 lists (head by head), one to four warps per query over up
-// to 512 lists when k <= 16 (also head by head), and the block merge of
-// merge.cuh (one CTA per query) otherwise; for unsorted lists (buffered
-// tensor-core lists, k > 32) one warp per query over all their keys.
+// Four merges: for unsorted lists (buffered tensor-core lists, k > 32) and
+// for sorted lists of at most 32 keys merged into k > 32, one warp per query
+// over all their keys; otherwise for sorted lists, by list count and k, one
+// warp per query over at most 32 lists (head by head), one to four warps per
+// query over up to 512 lists when k <= 16 (also head by head), and the block
+// merge of merge.cuh (one CTA per query).
 #include "merge.cuh"
 
 namespace oprag {
@@ -210,10 +211,12 @@ merge_small_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
   }
 }
 
-// Unsorted lists (ListSet::counts), k > 32: one warp per query.  The warp
+// Unsorted lists (ListSet::counts), k > 32, and short sorted lists merged
+// into k > 32 (read whole, as if unsorted): one warp per query.  The warp
 // scans the query's list counts into offsets in shared memory, reads the
-// concatenated keys 32 x kUnsortedLoads at a time (each key finds its list
-// by binary search over the offsets), drops keys below the counted floor and
+// concatenated keys 32 x kUnsortedLoads at a time (a lane's keys come in
+// increasing order, so it finds each key's list by moving a cursor forward
+// over the offsets, rarely more than one step), drops keys below the counted floor and
 // keeps the rest in a WarpMerger, whose buffer is sorted only when it fills
 // up and once at the end.  A good floor leaves a few hundred keys of the
 // several thousand read, so a query usually costs one sort; the warps of
@@ -243,7 +246,10 @@ merge_unsorted_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
   const int np = merge_list_count(ls, tile);
   const int offs_len = (ls.P + 4) / 4 * 4;
   int* offs = reinterpret_cast<int*>(smem_u + kUnsortedWarps * kCap) + warp * offs_len;
-  const int* cnt = ls.counts + static_cast<int64_t>(tile) * ls.P * ls.TH + row;
+  const int* cnt = ls.counts != nullptr
+                       ? ls.counts + static_cast<int64_t>(tile) * ls.P * ls.TH + row
+                       : nullptr;
+  const int fixed = min(ls.klen, ls.stride);     // keys of a sorted list
   const uint64_t* base = ls.keys + (static_cast<int64_t>(tile) * ls.P * ls.TH + row) * ls.stride;
   const int64_t list_step = static_cast<int64_t>(ls.TH) * ls.stride;
 
@@ -251,7 +257,9 @@ merge_unsorted_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
   int total = 0;
   for (int p0 = 0; p0 < np; p0 += 32) {
     const int p = p0 + lane;
-    const int c = p < np ? max(0, min(cnt[static_cast<int64_t>(p) * ls.TH], ls.stride)) : 0;
+    const int c = p >= np          ? 0
+                  : cnt == nullptr ? fixed
+                                   : max(0, min(cnt[static_cast<int64_t>(p) * ls.TH], ls.stride));
     int incl = c;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -261,11 +269,13 @@ merge_unsorted_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
     if (p < np) offs[p] = total + incl - c;
     total += __shfl_sync(0xffffffffu, incl, 31);
   }
+  if (lane == 0) offs[np] = total;
   __syncwarp();
 
   WarpMerger<KP> m;
   m.init(smem_u + warp * kCap, k);
   m.worst = merge_floor_key(ls, qi, k);
+  int cur = 0;      // this lane's list: offs[cur] <= its next key's index
   for (int g = 0; g < total; g += 32 * kUnsortedLoads) {
     uint64_t key[kUnsortedLoads];
 #pragma unroll
@@ -273,13 +283,10 @@ merge_unsorted_kernel(ListSet ls, int q, int k, int64_t* __restrict__ out_ids,
       const int i = g + u * 32 + lane;
       key[u] = kEmptyKey;
       if (i < total) {
-        // the last list p with offs[p] <= i (it holds key i - offs[p])
-        int p0 = 0, p1 = np - 1;
-        while (p0 < p1) {
-          const int mid = (p0 + p1 + 1) >> 1;
-          if (offs[mid] <= i) p0 = mid; else p1 = mid - 1;
-        }
-        key[u] = base[p0 * list_step + (i - offs[p0])];
+        // the list holding key i: the last p with offs[p] <= i (offs[np] =
+        // total > i ends the walk)
+        while (offs[cur + 1] <= i) ++cur;
+        key[u] = base[cur * list_step + (i - offs[cur])];
       }
     }
 #pragma unroll
@@ -431,7 +438,10 @@ cudaError_t launch_merge_two(int q, const int64_t* a_ids, const float* a_sc, int
 cudaError_t launch_merge(const ListSet& ls, int q, int k, int64_t* out_ids, float* out_scores,
                          cudaStream_t st, float* kth_out, float* levels_out) {
   if (q <= 0) return cudaSuccess;
-  if (ls.counts != nullptr) {
+  // Unsorted lists, or sorted lists of at most 32 keys merged into more
+  // (the sampled first pass of a search with k > 32): one sort per query
+  // instead of k head-by-head rounds.
+  if (ls.counts != nullptr || (k > 32 && ls.klen <= 32 && ls.stride <= 32)) {
     if (k <= 64) return launch_unsorted_kp<64>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
     if (k <= 128)
       return launch_unsorted_kp<128>(ls, q, k, out_ids, out_scores, st, kth_out, levels_out);
