@@ -1431,6 +1431,7 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
           for (int c = 0; c < NC; ++c) {
             tmem_ld32_async(taddr + c * 32, ra);
             tmem_wait_ld(ra);
+            if (!kHybrid && c + 1 == NC) release_acc();   // see below
             process(ra, c, lb);
           }
         } else {
@@ -1445,12 +1446,11 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
           if (c + 2 < NC) tmem_ld32_async(taddr + (c + 2) * 32, ra);
           // The unit's last TMEM load has landed: hand the accumulator back
           // to the MMA before filtering the last chunk (the gathered hybrid
-          // form still reads its second accumulator while filtering).  Only
-          // for register lists: measured on GB300, 32768 x 1024 with 4096
-          // queries and k = 10 took 217.6 instead of 218.9 us a step, while
-          // 1M x 768 with 2048 queries and k = 100 (buffered lists, one
-          // epilogue set) took 2095 instead of 2081 us in the main pass.
-          if (!kHybrid && K <= 32 && c + 2 >= NC) release_acc();
+          // form still reads its second accumulator while filtering).
+          // Measured on GB300: 32768 x 1024 with 4096 queries and k = 10,
+          // 217.6 instead of 218.9 us a step; 1M x 768 with 2048 queries and
+          // k = 100, main pass 1835 instead of 1868 us.
+          if (!kHybrid && c + 2 >= NC) release_acc();
           process(rb, c + 1, lb);
         }
         }
