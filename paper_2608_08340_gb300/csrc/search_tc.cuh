@@ -679,6 +679,13 @@ __device__ __forceinline__ void cp_async8(void* dst, const void* src) {
                : "memory");
 }
 
+// 16 bytes, or 16 zero bytes when !in (nothing is read from src then).
+__device__ __forceinline__ void cp_async16_zfill(void* dst, const void* src, bool in) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_addr(dst)), "l"(src),
+               "r"(in ? 16 : 0)
+               : "memory");
+}
+
 __device__ __forceinline__ void cp_async_commit_wait_all() {
   asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
 }
@@ -1235,11 +1242,9 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
       if constexpr (K > 32) list.read_ahead();
       if (warp_live) {
         float inv_max = 0.f;
-        const float* brow = nullptr;
         if (kLex != kLexNone && act) {
           const float m = p.fu.bm25_max[j * kBlockM + row];
           inv_max = m > 0.f ? 1.f / m : 0.f;
-          if (kLex == kLexBlock) brow = p.fu.bm25 + static_cast<int64_t>(j * kBlockM + row) * p.fu.ld;
         }
         const uint32_t taddr = tmem_base + (static_cast<uint32_t>(eg * 32) << 16) +
                                static_cast<uint32_t>(acc * BN);
@@ -1256,23 +1261,40 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
           for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
           const int64_t id0 = id_base + c * 32;
           if constexpr (kLex == kLexBlock) {
+            // The warp's 32 rows x 32 columns of the BM25 block, copied row
+            // by row with cp.async (eight lanes per 128-byte row, four rows
+            // per round: a lane reading its own row would touch 32 lines per
+            // load) straight into the staging rows of the lanes that own the
+            // rows (the filter stages its candidates there only after this).
+            // Rows past the batch and columns past the block's width read as
+            // 0; columns past the corpus become -inf below.
+            float* wrows = stage_rows + (warp - 2) * 32 * 32;
+            const int sub = lane >> 3, part = lane & 7;
+            const int64_t col = id0 + part * 4;
+            int64_t qrow = static_cast<int64_t>(j) * kBlockM + eg * 32 + sub;
+            const float* src = p.fu.bm25 + qrow * p.fu.ld + col;
+            __syncwarp();                        // the staging rows' last readers are done
+#pragma unroll 1
+            for (int rr = sub; rr < 32; rr += 4) {
+              const bool in = qrow < p.q && col < p.fu.ld;
+              cp_async16_zfill(wrows + rr * 32 + ((part ^ (rr & 7)) << 2), in ? src : p.fu.bm25, in);
+              src += 4 * p.fu.ld;
+              qrow += 4;
+            }
+            cp_async_commit_wait_all();
+            __syncwarp();
             if (act) {
               const float a = p.fu.alpha, b1 = 1.f - p.fu.alpha;
-              if (id0 + 32 <= id_end) {
 #pragma unroll
-                for (int i = 0; i < 32; i += 4) {
-                  const float4 w = *reinterpret_cast<const float4*>(brow + id0 + i);
-                  v[i] = fmaf(a, v[i], b1 * (w.x * inv_max));
-                  v[i + 1] = fmaf(a, v[i + 1], b1 * (w.y * inv_max));
-                  v[i + 2] = fmaf(a, v[i + 2], b1 * (w.z * inv_max));
-                  v[i + 3] = fmaf(a, v[i + 3], b1 * (w.w * inv_max));
-                }
-              } else {
-#pragma unroll
-                for (int i = 0; i < 32; ++i)
-                  if (id0 + i < id_end) v[i] = fmaf(a, v[i], b1 * (brow[id0 + i] * inv_max));
+              for (int g = 0; g < 8; ++g) {
+                const float4 x = *reinterpret_cast<const float4*>(srow + ((g ^ swz) << 2));
+                v[4 * g] = fmaf(a, v[4 * g], b1 * (x.x * inv_max));
+                v[4 * g + 1] = fmaf(a, v[4 * g + 1], b1 * (x.y * inv_max));
+                v[4 * g + 2] = fmaf(a, v[4 * g + 2], b1 * (x.z * inv_max));
+                v[4 * g + 3] = fmaf(a, v[4 * g + 3], b1 * (x.w * inv_max));
               }
             }
+            __syncwarp();
           }
           if constexpr (kHybrid) {
             // head terms from the second accumulator, the other terms from
