@@ -131,6 +131,7 @@ struct TcPlan {
   int nt;          // corpus tiles
   int win;         // corpus tiles per L2 window
   int pmax;        // lists per query tile
+  int sets;        // lists each CTA keeps per query tile (its epilogue sets; 1 in dual mode)
   int tile_stride; // corpus tiles skipped between scanned tiles (1 = all)
   int stages;
   size_t smem;

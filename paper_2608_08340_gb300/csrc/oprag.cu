@@ -1457,12 +1457,10 @@ int oprag_plan_search(int64_t n, int32_t d, int32_t q, int32_t k, int32_t num_sm
                 (long long)n, d, q, k, num_sms);
   const SearchShape s{n, d, q, k};
   const TcPlan pl = tc_plan(s, num_sms, force_block_n, 1, force_pair, pair_capacity);
-  const int K = list_len_for(k);
   const int64_t v[13] = {pl.grid,  pl.block_n, pl.pair,  pl.dual ? 1 : 0,
                          pl.qt,    pl.uqt,     pl.nt,    pl.win,
                          pl.pmax,  pl.stages,  static_cast<int64_t>(pl.smem),
-                         static_cast<int64_t>(tc_scratch_bytes(s, pl)),
-                         pl.dual ? 1 : (K <= 16 ? 2 : 1)};
+                         static_cast<int64_t>(tc_scratch_bytes(s, pl)), pl.sets};
   for (int i = 0; i < 13; ++i) out[i] = v[i];
   return ok();
 }

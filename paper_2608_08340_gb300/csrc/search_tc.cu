@@ -135,7 +135,8 @@ TcPlan tc_plan(const SearchShape& s, int num_sms, int force_block_n, int tile_st
   for (int j = 0; j < pl.uqt; ++j)
     per_tile = std::max(per_tile, hi[j] - first_cta(j, pl.uqt, C) + 1);
   if (!ok) per_tile = C;  // not expected; every slot then gets a list per tile
-  pl.pmax = per_tile * (pl.dual ? 1 : epi_sets(list_len_for(s.k), s.fused_lex));
+  pl.sets = pl.dual ? 1 : epi_sets(list_len_for(s.k), s.fused_lex);
+  pl.pmax = per_tile * pl.sets;
   const int K = list_len_for(s.k);
   // Shared memory of the launch (the same sum as smem_for<BN, K, pair, dual>).
   const size_t b_stage = static_cast<size_t>(pair ? bn / 2 : bn) * 128;

@@ -64,6 +64,10 @@ def test_plan_fits_and_provisions_every_list(n, d, q, k, force):
         assert p["block_n"] == 128 and p["cluster"] == 1 and list_len(k) <= 16
     if p["cluster"] == 2:
         assert p["block_n"] == 256
+    # Lists per CTA and query tile: one per epilogue set (two for lists of
+    # 8-16 and for buffered lists, one for lists of 32), one in dual mode.
+    kl = list_len(k)
+    assert p["sets"] == (1 if p["dual"] else (2 if kl <= 16 or kl > 32 else 1))
     # Every (query tile, slot) the schedule produces owns a list slot.
     pairs, c = replay_slots(p)
     per_tile = p["pmax"] // p["sets"]
