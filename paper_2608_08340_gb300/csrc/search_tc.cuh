@@ -194,11 +194,14 @@ __host__ __device__ constexpr int lex_land_bytes(bool lex) {
   return lex ? 128 * kLexLandStride : 0;
 }
 
-template <int BN, bool kPair = false, bool kDual = false, bool kLex = false>
+// kExtra: further shared memory of the launch (the BM25 block form's second
+// staging tile per epilogue warp, block_land_bytes).
+template <int BN, bool kPair = false, bool kDual = false, bool kLex = false, int kExtra = 0>
 constexpr int stages_for() {
-  return (kSmemBudget - lex_land_bytes(kLex)) / (a_stage_bytes<kDual>() + b_stage_bytes<BN, kPair>()) > 8
+  return (kSmemBudget - lex_land_bytes(kLex) - kExtra) /
+                     (a_stage_bytes<kDual>() + b_stage_bytes<BN, kPair>()) > 8
              ? 8
-             : (kSmemBudget - lex_land_bytes(kLex)) /
+             : (kSmemBudget - lex_land_bytes(kLex) - kExtra) /
                    (a_stage_bytes<kDual>() + b_stage_bytes<BN, kPair>());
 }
 
@@ -206,12 +209,12 @@ constexpr int stages_for() {
 // that candidate columns can be read back by index.
 constexpr int kStageRowBytes = 32 * 4;
 
-template <int BN, int K, bool kPair = false, bool kDual = false, bool kLex = false>
+template <int BN, int K, bool kPair = false, bool kDual = false, bool kLex = false, int kExtra = 0>
 constexpr size_t smem_for() {
-  return static_cast<size_t>(stages_for<BN, kPair, kDual, kLex>()) *
+  return static_cast<size_t>(stages_for<BN, kPair, kDual, kLex, kExtra>()) *
              (a_stage_bytes<kDual>() + b_stage_bytes<BN, kPair>()) +
          static_cast<size_t>(epi_sets(K, kLex)) * 128 * kStageRowBytes + lex_land_bytes(kLex) +
-         1024 + 256;
+         kExtra + 1024 + 256;
 }
 
 // ----------------------------------------------------------------- PTX
@@ -686,6 +689,14 @@ __device__ __forceinline__ void cp_async16_zfill(void* dst, const void* src, boo
                : "memory");
 }
 
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+}
+
 __device__ __forceinline__ void cp_async_commit_wait_all() {
   asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
 }
@@ -888,6 +899,14 @@ struct LexCursor {
 // the epilogue adds the other terms from the postings (LexCursor) and fuses.
 constexpr int kLexNone = 0, kLexBlock = 1, kLexGather = 2;
 
+// The BM25 block form's second staging tile: 32 x 32 floats per epilogue
+// warp, so that the next chunk's copy of the block flies while one chunk is
+// filtered.
+template <int K, int L>
+constexpr int block_land_bytes() {
+  return L == kLexBlock ? epi_sets(K) * 128 * kStageRowBytes : 0;
+}
+
 template <int BN, int K, int kLex, bool kPair = false, bool kDual = false>
 __global__ void __launch_bounds__(threads_for(K, kLex == kLexGather), 1)
 tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_e,
@@ -899,7 +918,8 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
   constexpr bool kHybrid = kLex == kLexGather;   // the gathered form
   static_assert(!kHybrid || (!kPair && !kDual && BN == 128),
                 "the gathered hybrid search runs single CTAs on 128-row tiles");
-  constexpr int S = stages_for<BN, kPair, kDual, kHybrid>();
+  constexpr int kLand = block_land_bytes<K, kLex>();
+  constexpr int S = stages_for<BN, kPair, kDual, kHybrid, kLand>();
   constexpr uint32_t kAStage = a_stage_bytes<kDual>();
   constexpr uint32_t kBStageBytes = b_stage_bytes<BN, kPair>();
   constexpr uint32_t kTmemCols = (kDual ? 4 : 2) * BN * (kHybrid ? 2 : 1);
@@ -915,7 +935,8 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
   float* stage_rows = reinterpret_cast<float*>(sB + S * kBStageBytes);   // epilogue staging
   // hybrid: each epilogue thread's landing zone of the lexical copies
   unsigned char* lex_land = reinterpret_cast<unsigned char*>(stage_rows + kEpiSets * 128 * 32);
-  uint64_t* full = reinterpret_cast<uint64_t*>(lex_land + lex_land_bytes(kHybrid));
+  float* block_land = reinterpret_cast<float*>(lex_land + lex_land_bytes(kHybrid));
+  uint64_t* full = reinterpret_cast<uint64_t*>(reinterpret_cast<unsigned char*>(block_land) + kLand);
   uint64_t* empty = full + S;
   uint64_t* tfull = empty + S;
   uint64_t* tempty = tfull + 4;
@@ -1253,6 +1274,36 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         float* srow = stage_rows + ((warp - 2) * 32 + lane) * 32;
         const int swz = lane & 7;
         unsigned char* land = lex_land + ((warp - 2) * 32 + lane) * kLexLandStride;
+        // BM25 block form: the warp's 32 x 32 tile of the block for chunk c
+        // sits in the staging rows (c even) or in the second tile (c odd);
+        // the filter stages the chunk's candidates in the same tile, and the
+        // next chunk's copy goes to the other one while this one is filtered.
+        constexpr int NC = BN / 32;              // 32-column chunks of a unit
+        float* wtile[2] = {stage_rows + (warp - 2) * 32 * 32, block_land + (warp - 2) * 32 * 32};
+        auto row_of = [&](int c) -> float* {
+          return kLex == kLexBlock && (c & 1) ? wtile[1] + lane * 32 : srow;
+        };
+        int block_next = -1;     // chunk whose block tile is in flight (-1: none)
+        // Copies chunk c's tile row by row with cp.async (eight lanes per
+        // 128-byte row, four rows per round: a lane reading its own row would
+        // touch 32 lines per load) straight into the rows of the lanes that
+        // own the query rows.  Rows past the batch and columns past the
+        // block's width read as 0; columns past the corpus become -inf later.
+        auto copy_block = [&](int c) {
+          float* tile = wtile[c & 1];
+          const int sub = lane >> 3, part = lane & 7;
+          const int64_t col = id_base + c * 32 + part * 4;
+          int64_t qrow = static_cast<int64_t>(j) * kBlockM + eg * 32 + sub;
+          const float* src = p.fu.bm25 + qrow * p.fu.ld + col;
+#pragma unroll 1
+          for (int rr = sub; rr < 32; rr += 4) {
+            const bool in = qrow < p.q && col < p.fu.ld;
+            cp_async16_zfill(tile + rr * 32 + ((part ^ (rr & 7)) << 2), in ? src : p.fu.bm25, in);
+            src += 4 * p.fu.ld;
+            qrow += 4;
+          }
+          cp_async_commit();
+        };
         // Scores of one chunk (corpus rows id0 .. id0 + 31), fused with the
         // lexical part when hybrid, -inf past the end of the corpus.  Called
         // by every lane of a live warp (the TMEM load is warp-collective).
@@ -1261,40 +1312,28 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
           for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
           const int64_t id0 = id_base + c * 32;
           if constexpr (kLex == kLexBlock) {
-            // The warp's 32 rows x 32 columns of the BM25 block, copied row
-            // by row with cp.async (eight lanes per 128-byte row, four rows
-            // per round: a lane reading its own row would touch 32 lines per
-            // load) straight into the staging rows of the lanes that own the
-            // rows (the filter stages its candidates there only after this).
-            // Rows past the batch and columns past the block's width read as
-            // 0; columns past the corpus become -inf below.
-            float* wrows = stage_rows + (warp - 2) * 32 * 32;
-            const int sub = lane >> 3, part = lane & 7;
-            const int64_t col = id0 + part * 4;
-            int64_t qrow = static_cast<int64_t>(j) * kBlockM + eg * 32 + sub;
-            const float* src = p.fu.bm25 + qrow * p.fu.ld + col;
-            __syncwarp();                        // the staging rows' last readers are done
-#pragma unroll 1
-            for (int rr = sub; rr < 32; rr += 4) {
-              const bool in = qrow < p.q && col < p.fu.ld;
-              cp_async16_zfill(wrows + rr * 32 + ((part ^ (rr & 7)) << 2), in ? src : p.fu.bm25, in);
-              src += 4 * p.fu.ld;
-              qrow += 4;
+            if (block_next != c) {
+              __syncwarp();                      // the tile's last readers are done
+              copy_block(c);
             }
-            cp_async_commit_wait_all();
+            cp_async_wait_all();
             __syncwarp();
             if (act) {
               const float a = p.fu.alpha, b1 = 1.f - p.fu.alpha;
+              const float* row = row_of(c);
 #pragma unroll
               for (int g = 0; g < 8; ++g) {
-                const float4 x = *reinterpret_cast<const float4*>(srow + ((g ^ swz) << 2));
+                const float4 x = *reinterpret_cast<const float4*>(row + ((g ^ swz) << 2));
                 v[4 * g] = fmaf(a, v[4 * g], b1 * (x.x * inv_max));
                 v[4 * g + 1] = fmaf(a, v[4 * g + 1], b1 * (x.y * inv_max));
                 v[4 * g + 2] = fmaf(a, v[4 * g + 2], b1 * (x.z * inv_max));
                 v[4 * g + 3] = fmaf(a, v[4 * g + 3], b1 * (x.w * inv_max));
               }
             }
-            __syncwarp();
+            // The other tile's last users (the previous chunk's filter, which
+            // ends with a warp barrier) are done: start the next chunk's copy.
+            block_next = c + 1 < NC ? c + 1 : -1;
+            if (block_next >= 0) copy_block(block_next);
           }
           if constexpr (kHybrid) {
             // head terms from the second accumulator, the other terms from
@@ -1352,11 +1391,13 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
 #pragma unroll
               for (int i = 0; i < 32; ++i) part[i >> 3] |= (v[i] >= fl ? 1u : 0u) << i;
               mask = (part[0] | part[1]) | (part[2] | part[3]);
+              float* crow = row_of(c);
 #pragma unroll
               for (int g = 0; g < 8; ++g)
-                *reinterpret_cast<float4*>(srow + ((g ^ swz) << 2)) =
+                *reinterpret_cast<float4*>(crow + ((g ^ swz) << 2)) =
                     make_float4(v[4 * g], v[4 * g + 1], v[4 * g + 2], v[4 * g + 3]);
             }
+            const float* crow = row_of(c);
             // Warp-uniform number of rounds; each round takes the lowest
             // remaining candidate column of every lane (ids stay increasing)
             // and inserts it with the branch-free network, so rounds are
@@ -1367,13 +1408,12 @@ tc_search_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
               const int i = __ffs(mask) - 1;
               const bool has = mask != 0;
               mask &= mask - 1;
-              const float s = has ? srow[((((i & 31) >> 2) ^ swz) << 2) | (i & 3)] : -INFINITY;
+              const float s = has ? crow[((((i & 31) >> 2) ^ swz) << 2) | (i & 3)] : -INFINITY;
               list.insert(s, static_cast<uint32_t>(id0 + i));
             }
           }
           __syncwarp();
         };
-        constexpr int NC = BN / 32;
         static_assert(NC % 2 == 0, "chunks are processed in pairs");
         uint32_t ra[32], rb[32];
         float bound = -INFINITY;
@@ -1520,7 +1560,7 @@ struct TcMaps {
 // Pair mode: clusters of two CTAs; `grid` counts CTAs (even).
 template <int BN, int K, int L>
 cudaError_t launch_pair_variant(const TcMaps& m, const TcParams& prm, int grid, cudaStream_t st) {
-  constexpr size_t smem = smem_for<BN, K, true>();
+  constexpr size_t smem = smem_for<BN, K, true, false, false, block_land_bytes<K, L>()>();
   static bool configured = false;
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(tc_search_kernel<BN, K, L, true>,
@@ -1551,7 +1591,7 @@ int pair_capacity_query();
 template <int BN, int K, int L>
 cudaError_t launch_variant(const TcMaps& m, const TcParams& prm, int grid, cudaStream_t st) {
   constexpr bool g = L == kLexGather;
-  constexpr size_t smem = smem_for<BN, K, false, false, g>();
+  constexpr size_t smem = smem_for<BN, K, false, false, g, block_land_bytes<K, L>()>();
   static bool configured = false;
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(tc_search_kernel<BN, K, L>,
@@ -1567,7 +1607,7 @@ cudaError_t launch_variant(const TcMaps& m, const TcParams& prm, int grid, cudaS
 // Dual mode (two query tiles per unit); 128-row corpus tiles, lists of 8 or 16.
 template <int K, int L>
 cudaError_t launch_dual_variant(const TcMaps& m, const TcParams& prm, int grid, cudaStream_t st) {
-  constexpr size_t smem = smem_for<128, K, false, true>();
+  constexpr size_t smem = smem_for<128, K, false, true, false, block_land_bytes<K, L>()>();
   static bool configured = false;
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(tc_search_kernel<128, K, L, false, true>,
